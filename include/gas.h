@@ -1,0 +1,169 @@
+/*
+ * gas.h — geometry-aware FP8 attention scales on one GB300 (sm_103a).
+ *
+ * For every query head h of every layer l this library computes the spectral norm
+ *     sigma_{l,h} = || W^Q_h W^K_{g(h)}^T ||_2            (paper, Eq. 4 and Eq. 7)
+ * by implicit power iteration (Section 4.1, Algorithm 2): the d x d interaction
+ * matrix is never formed, and under grouped-query attention the shared key block
+ * W^K_g is read unexpanded (Section 4.2, Algorithm 3, Proposition 4.1).  From the
+ * per-head sigmas it evaluates the per-layer geometry-aware scale (Section 3.4, Eq. 15)
+ *     scale_l = alpha * max_h sigma_{l,h} * (d / sqrt(d_h)) / (eta_fp8 * R_max),
+ * with alpha >= alpha_min from Eq. 13 and the typicality gamma from Eq. 12.
+ *
+ * Conventions shared by every entry point
+ *  - Weights use the nn.Linear layout, bf16, row-major, one allocation per layer:
+ *      Wq[l] : [n_q  * d_h, d]   rows h*d_h .. h*d_h+d_h-1 are (W^Q_h)^T
+ *      Wk[l] : [n_kv * d_h, d]   rows g*d_h .. are (W^K_g)^T
+ *    Query head h uses KV group g(h) = h / (n_q / n_kv) (RepeatBlocks order,
+ *    Appendix F).  Each layer pointer must be 16-byte aligned.
+ *  - Vectors are fp32, [layers][n_q][d] contiguous, 16-byte aligned.
+ *  - The caller owns every buffer passed in.  The handle owns only its workspace
+ *    (device memory sized at gas_create) and cached TMA descriptors.
+ *  - Calls that take a stream are asynchronous and stream-ordered; the host checks
+ *    arguments synchronously and enqueues nothing on error.  `stream` is a
+ *    cudaStream_t (NULL = legacy default stream).
+ *  - No exceptions cross this boundary.  A handle is not thread-safe; concurrent
+ *    calls on one handle (or overlapping launches of one handle on two streams)
+ *    race on its workspace.
+ *  - Device-side failures (a bounded wait that ran out, a NaN/Inf sigma) set bits
+ *    in a device status word read by gas_get_device_status; kernels never trap
+ *    and never wait without a limit.
+ */
+#ifndef GAS_H_
+#define GAS_H_
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct gas_ctx *gas_handle;
+
+typedef enum {
+    GAS_OK = 0,
+    GAS_ERR_INVALID_ARG = 1,   /* null/misaligned pointer, bad count, gamma in (0,1] ... */
+    GAS_ERR_UNSUPPORTED = 2,   /* shape outside what the kernels implement */
+    GAS_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed (see gas_last_error) */
+    GAS_ERR_ALLOC = 4,         /* workspace allocation failed */
+    GAS_ERR_DEVICE_TIMEOUT = 5 /* a device-side bounded wait ran out (status word) */
+} gas_status;
+
+/* Device status word bits (gas_get_device_status). */
+#define GAS_DEV_NONFINITE_SIGMA 0x1  /* some sigma came out NaN or Inf */
+#define GAS_DEV_WAIT_TIMEOUT    0x2  /* a bounded mbarrier/flag wait gave up */
+
+/* Power-iteration back ends (gas_set_method). */
+#define GAS_METHOD_AUTO   0  /* library picks (Gram for every iteration count it supports) */
+#define GAS_METHOD_STREAM 1  /* per-iteration streaming matvec chain, Algorithm 2 literally */
+#define GAS_METHOD_GRAM   2  /* one weight pass to d_h x d_h Gram matrices, iterate in R^{d_h} */
+
+/*
+ * Create a handle for one model shape (the paper's Section 4 cost model
+ * O(n_q * d_h * d) per layer per iteration).
+ *   layers >= 1; d >= 8 and d % 8 == 0 (16-byte rows); n_q, n_kv >= 1 with
+ *   n_q % n_kv == 0; d_h in {64, 128}; group size n_q/n_kv <= 64 (d_h 128) or 32 (d_h 64).
+ * Allocates the device workspace on the current device (see gas_workspace_bytes).
+ * Errors: GAS_ERR_INVALID_ARG (out == NULL, non-positive sizes), GAS_ERR_UNSUPPORTED
+ * (shape limits above), GAS_ERR_ALLOC, GAS_ERR_CUDA.  *out is NULL on error.
+ */
+gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle *out);
+
+/* Free the workspace (synchronises the device first).  NULL is a no-op. */
+gas_status gas_destroy(gas_handle h);
+
+/* Bytes of device workspace the handle holds. */
+size_t gas_workspace_bytes(gas_handle h);
+
+/*
+ * Calibration constants used by gas_scales / gas_refresh (Sections 3.2, 3.4):
+ *   seq_len L (Eq. 12-13, default 1024), eta_fp8 (Eq. 15, default 0.8),
+ *   alpha_override > 0 replaces alpha_min (the paper's rounded 0.08/0.04/0.03/0.02
+ *   or an auto-alpha result, Section 3.5); <= 0 restores alpha_min.
+ * Errors: GAS_ERR_INVALID_ARG for seq_len < 1 or eta_fp8 outside (0, 1].
+ */
+gas_status gas_set_calibration(gas_handle h, int seq_len, double eta_fp8, double alpha_override);
+
+/* Select the power-iteration back end (GAS_METHOD_*). */
+gas_status gas_set_method(gas_handle h, int method);
+
+/*
+ * Per-head spectral norms by `iters` power iterations (Algorithm 2 per head; one
+ * iteration = u' = M v, sigma = ||u'||, u = u'/sigma, v' = M^T u, v = v'/||v'||;
+ * the reported sigma is the last iteration's ||M v_{k-1}||).
+ *   wq, wk : HOST arrays of `layers` DEVICE pointers to the bf16 Wq[l], Wk[l].
+ *   iters  : >= 1 (cold start: the paper uses 5; warm refresh: 1-2).
+ *   v_in   : device fp32 [layers][n_q][d] start vectors (any scale; a zero vector
+ *            gives sigma = 0 and v_out = 0).  Warm start: pass last call's v_out.
+ *   v_out  : device fp32, same shape, unit right singular vector estimates; may
+ *            alias v_in; NULL skips the write-back.
+ *   sigma  : device fp32 [layers][n_q].
+ * Errors: GAS_ERR_INVALID_ARG (NULL or misaligned pointers, iters < 1),
+ * GAS_ERR_CUDA (launch failure).
+ */
+gas_status gas_spectral_norms(gas_handle h, const void *const *wq, const void *const *wk,
+                              int iters, const float *v_in, float *v_out, float *sigma,
+                              void *stream);
+
+/*
+ * Per-layer scale (Eq. 15) from per-head sigmas: s[l] = alpha * max_h sigma[l][h] *
+ * (d / sqrt(d_h)) / (eta_fp8 * r_max).  N = layers * n_q heads enter Eq. 12-13.
+ *   gamma      : > 1 uses it; <= 0 solves Eq. 12 for the minimal gamma; (0, 1] is an error.
+ *   delta_star : target overflow probability, > 0 (paper: 1e-6).
+ *   r_max      : format maximum, > 0 (448 for E4M3).
+ *   sigma, s   : device fp32 [layers][n_q] in, [layers] out.
+ * A NaN sigma propagates into its layer's scale.
+ */
+gas_status gas_scales(gas_handle h, const float *sigma, double gamma, double delta_star,
+                      double r_max, float *s, void *stream);
+
+/*
+ * gas_spectral_norms followed by gas_scales, with the per-layer max and the
+ * scale evaluated inside the last power-iteration kernel (no separate pass).
+ * Arguments as above.
+ */
+gas_status gas_refresh(gas_handle h, const void *const *wq, const void *const *wk, int iters,
+                       const float *v_in, float *v_out, float *sigma, double gamma,
+                       double delta_star, double r_max, float *s, void *stream);
+
+/* Host helpers in float64: Eq. 12 (smallest gamma > 1; 1.0 if the bound holds for
+ * every gamma; NaN on invalid input) and Eq. 13 (alpha_min for a given gamma). */
+double gas_gamma_min(int d_h, long long n_heads_total, int seq_len, double delta_star);
+double gas_alpha_min(double gamma, int d, int d_h, long long n_heads_total, int seq_len,
+                     double delta_star);
+
+/* Gamma and alpha the handle would use for gas_scales with this gamma / delta*. */
+gas_status gas_resolve_calibration(gas_handle h, double gamma, double delta_star,
+                                   double *gamma_out, double *alpha_out);
+
+/* Message for the last error on this handle (or the last gas_create failure when h is NULL). */
+const char *gas_last_error(gas_handle h);
+const char *gas_status_string(gas_status s);
+
+/* Read (blocking: synchronises the device) and optionally clear the device status
+ * word (GAS_DEV_* bits).  Returns GAS_ERR_DEVICE_TIMEOUT when the timeout bit is set. */
+gas_status gas_get_device_status(gas_handle h, int *code, int clear);
+
+/* Number of kernel launches the last gas_spectral_norms / gas_refresh enqueued. */
+int gas_last_launch_count(gas_handle h);
+
+/*
+ * Diagnostic timing hook.  When events != NULL, every kernel that a later
+ * gas_spectral_norms / gas_refresh / gas_scales enqueues (in order, i = 0, 1, ...)
+ * is bracketed by cudaEventRecord(events[2i]) before and events[2i+1] after, on the
+ * call's stream, for the first n_events/2 kernels.  The events are caller-owned
+ * cudaEvent_t handles (created without cudaEventDisableTiming) and must outlive the
+ * calls; pass NULL / 0 to switch recording off.  Names of the kernels in launch order
+ * are available from gas_last_launch_name.
+ * Errors: GAS_ERR_INVALID_ARG for n_events < 0 or odd.
+ */
+gas_status gas_set_launch_events(gas_handle h, void *const *events, int n_events);
+
+/* Kernel name of launch i of the last call ("" when out of range). */
+const char *gas_last_launch_name(gas_handle h, int i);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GAS_H_ */

@@ -1,0 +1,271 @@
+"""Python binding of ``libgas.so`` (include/gas.h): argument marshalling only.
+
+Per-head spectral norms sigma_{l,h} = ||W^Q_h W^K_{g(h)}^T||_2 by implicit power
+iteration (paper Section 4, Algorithms 2-3) and per-layer geometry-aware FP8 scales
+(Section 3.4, Eq. 15), all computed by the CUDA kernels of the library.  PyTorch only
+supplies device memory and the current stream.  There is no fallback: if the library
+cannot be loaded every call raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from typing import List, Optional, Sequence
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libgas.so")
+HEADER = os.path.join(os.path.dirname(HERE), "include", "gas.h")
+
+GAS_OK = 0
+GAS_ERR_INVALID_ARG = 1
+GAS_ERR_UNSUPPORTED = 2
+GAS_ERR_CUDA = 3
+GAS_ERR_ALLOC = 4
+GAS_ERR_DEVICE_TIMEOUT = 5
+
+GAS_DEV_NONFINITE_SIGMA = 0x1
+GAS_DEV_WAIT_TIMEOUT = 0x2
+
+METHOD_AUTO = 0
+METHOD_STREAM = 1
+METHOD_GRAM = 2
+METHODS = {"auto": METHOD_AUTO, "stream": METHOD_STREAM, "gram": METHOD_GRAM}
+
+E4M3_MAX = 448.0
+
+
+class GasError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{_status_name(status)}: {msg}")
+        self.status = status
+
+
+_lib = None
+
+
+def _status_name(s: int) -> str:
+    return {0: "GAS_OK", 1: "GAS_ERR_INVALID_ARG", 2: "GAS_ERR_UNSUPPORTED", 3: "GAS_ERR_CUDA",
+            4: "GAS_ERR_ALLOC", 5: "GAS_ERR_DEVICE_TIMEOUT"}.get(s, f"status {s}")
+
+
+def build(force: bool = False) -> str:
+    from .build import build as _build
+    return _build(force=force)
+
+
+def exported_names() -> List[str]:
+    """Function names declared in include/gas.h."""
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return re.findall(r"\b(gas_[a-z_]+)\s*\(", src)
+
+
+def load(path: str = LIB_PATH):
+    """Load the library (raises OSError if it is missing: no fallback path exists)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise OSError(f"{path} not found: build it with python -m paper_2602_18851_gb300.build")
+    lib = ctypes.CDLL(path)
+    vp, c_int, c_double, c_ll = ctypes.c_void_p, ctypes.c_int, ctypes.c_double, ctypes.c_longlong
+    lib.gas_create.argtypes = [c_int] * 5 + [ctypes.POINTER(vp)]
+    lib.gas_destroy.argtypes = [vp]
+    lib.gas_workspace_bytes.argtypes = [vp]
+    lib.gas_workspace_bytes.restype = ctypes.c_size_t
+    lib.gas_set_calibration.argtypes = [vp, c_int, c_double, c_double]
+    lib.gas_set_method.argtypes = [vp, c_int]
+    lib.gas_spectral_norms.argtypes = [vp, vp, vp, c_int, vp, vp, vp, vp]
+    lib.gas_scales.argtypes = [vp, vp, c_double, c_double, c_double, vp, vp]
+    lib.gas_refresh.argtypes = [vp, vp, vp, c_int, vp, vp, vp, c_double, c_double, c_double, vp, vp]
+    lib.gas_gamma_min.argtypes = [c_int, c_ll, c_int, c_double]
+    lib.gas_gamma_min.restype = c_double
+    lib.gas_alpha_min.argtypes = [c_double, c_int, c_int, c_ll, c_int, c_double]
+    lib.gas_alpha_min.restype = c_double
+    lib.gas_resolve_calibration.argtypes = [vp, c_double, c_double, ctypes.POINTER(c_double),
+                                            ctypes.POINTER(c_double)]
+    lib.gas_last_error.argtypes = [vp]
+    lib.gas_last_error.restype = ctypes.c_char_p
+    lib.gas_status_string.argtypes = [c_int]
+    lib.gas_status_string.restype = ctypes.c_char_p
+    lib.gas_get_device_status.argtypes = [vp, ctypes.POINTER(c_int), c_int]
+    lib.gas_last_launch_count.argtypes = [vp]
+    lib.gas_set_launch_events.argtypes = [vp, vp, c_int]
+    lib.gas_last_launch_name.argtypes = [vp, c_int]
+    lib.gas_last_launch_name.restype = ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+def _check(st: int, h=None):
+    if st != GAS_OK:
+        msg = load().gas_last_error(h)
+        raise GasError(st, (msg or b"").decode())
+
+
+def gamma_min(d_h: int, n_heads_total: int, seq_len: int = 1024, delta_star: float = 1e-6) -> float:
+    """Eq. 12: smallest gamma > 1 with gamma - 1 - ln gamma >= (2/d_h) ln(2 N L / delta*)."""
+    return load().gas_gamma_min(int(d_h), int(n_heads_total), int(seq_len), float(delta_star))
+
+
+def alpha_min(gamma: float, d: int, d_h: int, n_heads_total: int, seq_len: int = 1024,
+              delta_star: float = 1e-6) -> float:
+    """Eq. 13: sqrt(2 gamma d_h)/d * sqrt(ln(4 N L^2 / delta*))."""
+    return load().gas_alpha_min(float(gamma), int(d), int(d_h), int(n_heads_total), int(seq_len),
+                                float(delta_star))
+
+
+def _ptr_array(tensors: Sequence[torch.Tensor], rows: int, d: int, name: str):
+    arr = (ctypes.c_void_p * len(tensors))()
+    for i, t in enumerate(tensors):
+        if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name}[{i}] must be a contiguous CUDA bfloat16 tensor")
+        if tuple(t.shape) != (rows, d):
+            raise ValueError(f"{name}[{i}] has shape {tuple(t.shape)}, expected {(rows, d)}")
+        arr[i] = t.data_ptr()
+    return arr
+
+
+def _stream_ptr(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+class Handle:
+    """One model shape (layers, d, n_q, n_kv, d_h) and its device workspace."""
+
+    def __init__(self, layers: int, d: int, n_q: int, n_kv: int, d_h: int):
+        lib = load()
+        self.layers, self.d, self.n_q, self.n_kv, self.d_h = layers, d, n_q, n_kv, d_h
+        h = ctypes.c_void_p()
+        _check(lib.gas_create(layers, d, n_q, n_kv, d_h, ctypes.byref(h)), None)
+        self._h = h
+
+    # -- lifetime --------------------------------------------------------------------
+    def close(self):
+        if getattr(self, "_h", None):
+            load().gas_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    # -- configuration -----------------------------------------------------------------
+    @property
+    def workspace_bytes(self) -> int:
+        return int(load().gas_workspace_bytes(self._h))
+
+    def set_calibration(self, seq_len: int = 1024, eta_fp8: float = 0.8, alpha_override: float = 0.0):
+        _check(load().gas_set_calibration(self._h, int(seq_len), float(eta_fp8), float(alpha_override)),
+               self._h)
+
+    def set_method(self, method):
+        m = METHODS[method] if isinstance(method, str) else int(method)
+        _check(load().gas_set_method(self._h, m), self._h)
+
+    def resolve_calibration(self, gamma: float = 0.0, delta_star: float = 1e-6):
+        g, a = ctypes.c_double(), ctypes.c_double()
+        _check(load().gas_resolve_calibration(self._h, float(gamma), float(delta_star), ctypes.byref(g),
+                                              ctypes.byref(a)), self._h)
+        return g.value, a.value
+
+    @property
+    def last_launch_count(self) -> int:
+        return int(load().gas_last_launch_count(self._h))
+
+    def last_launch_names(self) -> List[str]:
+        lib = load()
+        return [lib.gas_last_launch_name(self._h, i).decode() for i in range(self.last_launch_count)]
+
+    def set_launch_events(self, events: Optional[Sequence[torch.cuda.Event]]):
+        """Bracket each library kernel i of later calls with events[2i] / events[2i+1]."""
+        self._events = list(events) if events else []
+        if not self._events:
+            _check(load().gas_set_launch_events(self._h, None, 0), self._h)
+            return
+        for e in self._events:
+            if e.cuda_event == 0:  # torch creates the CUDA event lazily
+                e.record()
+        arr = (ctypes.c_void_p * len(self._events))(*[e.cuda_event for e in self._events])
+        _check(load().gas_set_launch_events(self._h, arr, len(self._events)), self._h)
+
+    def device_status(self, clear: bool = False) -> int:
+        code = ctypes.c_int()
+        st = load().gas_get_device_status(self._h, ctypes.byref(code), 1 if clear else 0)
+        if st not in (GAS_OK, GAS_ERR_DEVICE_TIMEOUT):
+            _check(st, self._h)
+        return code.value
+
+    # -- compute -------------------------------------------------------------------------
+    def _vec_args(self, v_in, v_out, sigma, device):
+        shape = (self.layers, self.n_q, self.d)
+        if v_in.dtype != torch.float32 or tuple(v_in.shape) != shape or not v_in.is_contiguous():
+            raise ValueError(f"v_in must be a contiguous float32 tensor of shape {shape}")
+        if sigma is None:
+            sigma = torch.empty(self.layers, self.n_q, device=device, dtype=torch.float32)
+        return v_out, sigma
+
+    def spectral_norms(self, wq: Sequence[torch.Tensor], wk: Sequence[torch.Tensor], iters: int,
+                       v_in: torch.Tensor, v_out: Optional[torch.Tensor] = None,
+                       sigma: Optional[torch.Tensor] = None, write_back: bool = True, stream=None):
+        """sigma[l,h] after `iters` power iterations from v_in; v_out the unit right
+        singular vector estimates (warm start for the next call).  Returns (sigma, v_out)."""
+        qa = _ptr_array(wq, self.n_q * self.d_h, self.d, "wq")
+        ka = _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk")
+        if v_out is None and write_back:
+            v_out = torch.empty_like(v_in)
+        v_out, sigma = self._vec_args(v_in, v_out, sigma, v_in.device)
+        st = load().gas_spectral_norms(self._h, qa, ka, int(iters), v_in.data_ptr(),
+                                       v_out.data_ptr() if v_out is not None else None,
+                                       sigma.data_ptr(), _stream_ptr(stream))
+        _check(st, self._h)
+        return sigma, v_out
+
+    def scales(self, sigma: torch.Tensor, gamma: float = 0.0, delta_star: float = 1e-6,
+               r_max: float = E4M3_MAX, s: Optional[torch.Tensor] = None, stream=None):
+        """Per-layer scale (Eq. 15) from per-head sigmas."""
+        if s is None:
+            s = torch.empty(self.layers, device=sigma.device, dtype=torch.float32)
+        st = load().gas_scales(self._h, sigma.data_ptr(), float(gamma), float(delta_star), float(r_max),
+                               s.data_ptr(), _stream_ptr(stream))
+        _check(st, self._h)
+        return s
+
+    def refresh(self, wq, wk, iters: int, v_in: torch.Tensor, v_out: Optional[torch.Tensor] = None,
+                sigma: Optional[torch.Tensor] = None, s: Optional[torch.Tensor] = None,
+                gamma: float = 0.0, delta_star: float = 1e-6, r_max: float = E4M3_MAX,
+                write_back: bool = True, stream=None):
+        """Spectral norms and per-layer scales in one call.  Returns (sigma, s, v_out)."""
+        qa = _ptr_array(wq, self.n_q * self.d_h, self.d, "wq")
+        ka = _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk")
+        if v_out is None and write_back:
+            v_out = torch.empty_like(v_in)
+        v_out, sigma = self._vec_args(v_in, v_out, sigma, v_in.device)
+        if s is None:
+            s = torch.empty(self.layers, device=v_in.device, dtype=torch.float32)
+        st = load().gas_refresh(self._h, qa, ka, int(iters), v_in.data_ptr(),
+                                v_out.data_ptr() if v_out is not None else None, sigma.data_ptr(),
+                                float(gamma), float(delta_star), float(r_max), s.data_ptr(),
+                                _stream_ptr(stream))
+        _check(st, self._h)
+        return sigma, s, v_out
+
+
+__all__ = ["Handle", "GasError", "load", "build", "gamma_min", "alpha_min", "exported_names",
+           "METHOD_AUTO", "METHOD_STREAM", "METHOD_GRAM", "E4M3_MAX", "LIB_PATH"]

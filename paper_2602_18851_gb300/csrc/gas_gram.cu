@@ -1,0 +1,411 @@
+// Gram back end: the same power iteration as Algorithm 2, moved into R^{d_h}.
+//
+// For head h with A = A_h = (W^Q_h)^T and B = B_g = (W^K_g)^T (both d_h x d), a unit v
+// and z = B v, one iteration of Algorithm 2 is, exactly,
+//   u' = A^T z,  ||u'||^2 = z^T (A A^T) z,  y = A u = (A A^T) z / ||u'||,
+//   v' = B^T y,  ||v'||^2 = y^T (B B^T) y,  z_next = B v = (B B^T) y / ||v'||.
+// So with the d_h x d_h Gram matrices G_Q = A A^T and G_K = B B^T the k iterations need
+// no further weight traffic: one pass over every A_h and B_g (tensor cores), k
+// iterations on 128 x 128 matrices (CUDA cores), and one more pass over B_g for the
+// write-back v_out = B^T y / ||v'||.
+//
+//   prep_v_kernel   v / ||v|| split into bf16 hi + lo rows (the tensor-core operand for z0)
+//   gram_kernel     persistent, warp-specialised: TMA -> smem ring -> tcgen05.mma into
+//                   TMEM; G = X X^T for every 128-row weight tile and, on key tiles,
+//                   Z = X [v_hi; v_lo]^T (z0 = B v in ~16-bit-mantissa precision)
+//   iterate_kernel  k iterations per head in R^{d_h} from G_Q, G_K, z0; sigma, y/||v'||,
+//                   fused per-layer scale (Eq. 15)
+// The write-back reuses the streaming K pass (gas_stream.cu).
+
+#include "gas_device.cuh"
+
+namespace gas {
+
+namespace {
+
+constexpr int kGramThreads = 192;  // warp 0 TMA producer, warp 1 MMA issuer, warps 2-5 epilogue
+constexpr uint32_t kTileBytes = 128u * 64u * 2u;  // one 128-row x 64-column bf16 box
+constexpr int kSmemBudget = 232448;               // 227 KB opt-in dynamic shared memory
+constexpr int kSmemReserve = 2048;                // alignment slack + barriers
+
+template <int NZ>
+struct GramCfg {
+  static constexpr uint32_t kVBytes = static_cast<uint32_t>(NZ) * 64u * 2u;
+  static constexpr uint32_t kStageBytes = kTileBytes + kVBytes;
+  static constexpr int kStages = (kSmemBudget - kSmemReserve) / static_cast<int>(kStageBytes);
+  static constexpr size_t kSmem = static_cast<size_t>(kStages) * kStageBytes + kSmemReserve;
+  static_assert(kStages >= 3, "ring too shallow");
+  static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
+};
+
+// ---- v / ||v|| as bf16 hi + lo rows ---------------------------------------------------
+// Row layout of one key tile's operand (nz rows): group gi of the tile owns rows
+// gi*2G .. gi*2G+2G-1; head j of the group has its hi part at gi*2G + j and its lo
+// part at gi*2G + G + j.  Padding rows stay zero (cleared at handle creation).
+__global__ void __launch_bounds__(256) prep_v_kernel(const __grid_constant__ PrepArgs a) {
+  const Shape& s = a.s;
+  const size_t hidx = blockIdx.x;
+  const int l = static_cast<int>(hidx / s.nq), h = static_cast<int>(hidx % s.nq);
+  const int g = h / s.G, j = h % s.G;
+  const int tk = (g * s.dh) / 128, gi = ((g * s.dh) % 128) / s.dh;
+  const float* v = a.v_in + hidx * s.d;
+  __shared__ float wsum[8];
+  float n2 = 0.0f;
+  for (int c = threadIdx.x * 4; c < s.d; c += blockDim.x * 4) {
+    const float4 x = *reinterpret_cast<const float4*>(v + c);
+    n2 = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, n2))));
+  }
+  n2 = warp_sum(n2);
+  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = n2;
+  __syncthreads();
+  float tot = 0.0f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) tot += wsum[w];
+  const float inv = safe_inv_sqrt(tot);
+  const size_t base = (static_cast<size_t>(l) * s.tiles_k + tk) * s.nz;
+  uint16_t* hi_row = a.vhl + (base + gi * 2 * s.G + j) * s.d;
+  uint16_t* lo_row = a.vhl + (base + gi * 2 * s.G + s.G + j) * s.d;
+  for (int c = threadIdx.x * 8; c < s.d; c += blockDim.x * 8) {
+    const float4 x0 = *reinterpret_cast<const float4*>(v + c);
+    const float4 x1 = *reinterpret_cast<const float4*>(v + c + 4);
+    const float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+    uint32_t hb[8], lb[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float xn = xv[e] * inv;
+      hb[e] = f32_to_bf16_bits(xn);
+      lb[e] = f32_to_bf16_bits(xn - __uint_as_float(hb[e] << 16));
+    }
+    *reinterpret_cast<uint4*>(hi_row + c) =
+        make_uint4(hb[0] | (hb[1] << 16), hb[2] | (hb[3] << 16), hb[4] | (hb[5] << 16), hb[6] | (hb[7] << 16));
+    *reinterpret_cast<uint4*>(lo_row + c) =
+        make_uint4(lb[0] | (lb[1] << 16), lb[2] | (lb[3] << 16), lb[4] | (lb[5] << 16), lb[6] | (lb[7] << 16));
+  }
+  if (a.s_zero != nullptr && h == 0 && threadIdx.x == 0) a.s_zero[l] = 0.0f;
+}
+
+// ---- tcgen05 Gram kernel -------------------------------------------------------------
+struct TileRef {
+  int layer, is_k, idx;
+};
+
+__device__ __forceinline__ TileRef decode_tile(const Shape& s, int t) {
+  const int tpl = s.tiles_k + s.tiles_q;
+  TileRef r;
+  r.layer = t / tpl;
+  const int rem = t - r.layer * tpl;
+  r.is_k = rem < s.tiles_k;
+  r.idx = r.is_k ? rem : rem - s.tiles_k;
+  return r;
+}
+
+template <int NZ>
+__global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_constant__ GramArgs a) {
+  using Cfg = GramCfg<NZ>;
+  constexpr int S = Cfg::kStages;
+  constexpr uint32_t SB = Cfg::kStageBytes;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * SB);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + S;
+  uint64_t* accf = bars + 2 * S;
+  uint64_t* acce = accf + 2;
+  uint64_t* done = acce + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int no_abort_flag = 0;
+
+  const Shape& s = a.s;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < S; ++i) {
+      mbar_init(smem_u32(&full[i]), 1);
+      mbar_init(smem_u32(&empty[i]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&accf[i]), 1);
+      mbar_init(smem_u32(&acce[i]), 128);
+    }
+    mbar_init(smem_u32(done), 1);
+    *abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int T = s.L * (s.tiles_k + s.tiles_q);
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      const uint64_t pol = l2_policy_evict_first();
+      uint32_t issued = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
+        const TileRef tr = decode_tile(s, t);
+        const CUtensorMap* map = tr.is_k ? &a.maps_k[tr.layer] : &a.maps_q[tr.layer];
+        const int row0 = tr.idx * 128;
+        const int vrow0 = (tr.layer * s.tiles_k + tr.idx) * NZ;
+        for (int kc = 0; kc < s.nkc; ++kc) {
+          const uint32_t st = issued % S, ph = (issued / S) & 1u;
+          if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1u, abort, a.status)) { ok = false; break; }
+          const uint32_t sx = smem_u32(smem + st * SB);
+          const uint32_t fb = smem_u32(&full[st]);
+          mbar_arrive_expect_tx(fb, tr.is_k ? SB : kTileBytes);
+          tma_load_2d(sx, map, fb, kc * 64, row0, pol);
+          if (tr.is_k) tma_load_2d(sx + kTileBytes, a.map_v, fb, kc * 64, vrow0, pol);
+          ++issued;
+        }
+      }
+      // Every copy still in flight targets this CTA's shared memory: wait for them to land.
+      const uint32_t first = issued > static_cast<uint32_t>(S) ? issued - S : 0u;
+      for (uint32_t i = first; i < issued; ++i)
+        mbar_wait(smem_u32(&full[i % S]), (i / S) & 1u, &no_abort_flag, a.status);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer (one thread) ----------------
+    if (lane == 0) {
+      constexpr uint32_t idG = idesc_bf16_f32(128, 128);
+      constexpr uint32_t idZ = idesc_bf16_f32(128, NZ);
+      uint32_t consumed = 0, tc = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
+        const TileRef tr = decode_tile(s, t);
+        const uint32_t acc = tc & 1u, aph = (tc >> 1) & 1u;
+        if (!mbar_wait(smem_u32(&acce[acc]), aph ^ 1u, abort, a.status)) break;
+        tc_fence_after();
+        const uint32_t dG = tmem + acc * 128u;
+        const uint32_t dZ = tmem + 256u + acc * static_cast<uint32_t>(NZ);
+        for (int kc = 0; kc < s.nkc; ++kc) {
+          const uint32_t st = consumed % S, ph = (consumed / S) & 1u;
+          if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sx = smem_u32(smem + st * SB);
+          const uint64_t ad = desc_kmajor_sw128(sx);
+          const uint64_t vd = desc_kmajor_sw128(sx + kTileBytes);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const uint32_t accum = (kc | k) != 0 ? 1u : 0u;
+            umma_bf16(dG, ad + 2u * k, ad + 2u * k, idG, accum);
+            if (tr.is_k) umma_bf16(dZ, ad + 2u * k, vd + 2u * k, idZ, accum);
+          }
+          umma_commit(smem_u32(&empty[st]));
+          ++consumed;
+        }
+        if (!ok) break;
+        umma_commit(smem_u32(&accf[acc]));
+        ++tc;
+      }
+      // Retire every MMA before tensor memory and shared memory go away.
+      umma_commit(smem_u32(done));
+      mbar_wait(smem_u32(done), 0u, &no_abort_flag, a.status);
+    }
+  } else {
+    // ---------------- epilogue: TMEM -> global ----------------
+    const int q = warp & 3;  // tcgen05.ld: warp w may read TMEM lanes 32*(w%4) .. +31
+    const int row = q * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const int gpt = 128 / s.dh;
+    uint32_t tc = 0;
+    for (int t = blockIdx.x; t < T; t += gridDim.x) {
+      const TileRef tr = decode_tile(s, t);
+      const uint32_t acc = tc & 1u, aph = (tc >> 1) & 1u;
+      const bool got = mbar_wait(smem_u32(&accf[acc]), aph, abort, a.status);
+      __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the per-lane wait
+      if (!__all_sync(0xFFFFFFFFu, got)) break;
+      tc_fence_after();
+      float* Gout = (tr.is_k ? a.gk : a.gq) +
+                    (static_cast<size_t>(tr.layer) * (tr.is_k ? s.tiles_k : s.tiles_q) + tr.idx) * 16384u;
+#pragma unroll 1
+      for (int c0 = 0; c0 < 128; c0 += 16) {
+        uint32_t r[16];
+        tmem_ld16(tmem + lane_off + acc * 128u + c0, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) Gout[(c0 + jj) * 128 + row] = __uint_as_float(r[jj]);
+      }
+      if (tr.is_k) {
+        const int gi = row / s.dh, i = row % s.dh;
+        const int g = tr.idx * gpt + gi;
+        const int twoG = 2 * s.G;
+#pragma unroll 1
+        for (int c0 = 0; c0 < NZ; c0 += 16) {
+          uint32_t r[16];
+          tmem_ld16(tmem + lane_off + 256u + acc * static_cast<uint32_t>(NZ) + c0, r);
+          tmem_ld_wait();
+#pragma unroll
+          for (int jj = 0; jj < 16; ++jj) {
+            const int rel = c0 + jj - gi * twoG;
+            if (g < s.nkv && rel >= 0 && rel < twoG) {
+              const int half = rel >= s.G ? 1 : 0;
+              const int head = g * s.G + rel - half * s.G;
+              a.z0[((static_cast<size_t>(tr.layer) * s.nq + head) * 2 + half) * s.dh + i] =
+                  __uint_as_float(r[jj]);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(smem_u32(&acce[acc]));
+      ++tc;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ---- k power iterations per head in R^{d_h} -------------------------------------------
+// 256 threads hold G_Q and G_K in registers: warp w owns rows [w*DH/8, (w+1)*DH/8),
+// lane l owns columns [l*DH/32, (l+1)*DH/32).  A matvec is 64 (d_h 128) FMAs per
+// thread, a 16-shuffle transpose reduction per warp and one shared-memory exchange.
+template <int DH>
+__global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ IterArgs a) {
+  constexpr int RPW = DH / 8;
+  constexpr int CPL = DH / 32;
+  const Shape& s = a.s;
+  const size_t hidx = blockIdx.x;
+  const int l = static_cast<int>(hidx / s.nq), h = static_cast<int>(hidx % s.nq);
+  const int g = h / s.G;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int oq = (h * DH) % 128, ok = (g * DH) % 128;
+  const float* GQ = a.gq + (static_cast<size_t>(l) * s.tiles_q + (h * DH) / 128) * 16384u + oq * 128 + oq;
+  const float* GK = a.gk + (static_cast<size_t>(l) * s.tiles_k + (g * DH) / 128) * 16384u + ok * 128 + ok;
+
+  float gq[RPW][CPL], gk[RPW][CPL];
+#pragma unroll
+  for (int rr = 0; rr < RPW; ++rr) {
+    const int r = warp * RPW + rr;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) {
+      gq[rr][c] = __ldg(GQ + r * 128 + lane * CPL + c);
+      gk[rr][c] = __ldg(GK + r * 128 + lane * CPL + c);
+    }
+  }
+  __shared__ float zs[DH], ts[DH], ws[DH];
+  if (tid < DH) zs[tid] = a.z0[(hidx * 2 + 0) * DH + tid] + a.z0[(hidx * 2 + 1) * DH + tid];
+  __syncthreads();
+  float z[CPL], y[CPL];
+#pragma unroll
+  for (int c = 0; c < CPL; ++c) z[c] = zs[lane * CPL + c];
+  float sigma = 0.0f, inv_n = 0.0f;
+  for (int it = 0; it < a.iters; ++it) {
+    // t = G_Q z  (= A u');  sigma^2 = z . t (= ||u'||^2);  y = t / sigma (= A u)
+    float part[RPW];
+#pragma unroll
+    for (int rr = 0; rr < RPW; ++rr) {
+      float acc = 0.0f;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) acc = fmaf(gq[rr][c], z[c], acc);
+      part[rr] = acc;
+    }
+    int idx;
+    float red = warp_transpose_reduce<RPW>(part, lane, idx);
+    if (transpose_reduce_writer<RPW>(lane)) ts[warp * RPW + idx] = red;
+    __syncthreads();
+    float t[CPL], s2 = 0.0f;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) {
+      t[c] = ts[lane * CPL + c];
+      s2 = fmaf(z[c], t[c], s2);
+    }
+    s2 = fmaxf(warp_sum(s2), 0.0f);
+    sigma = sqrtf(s2);
+    const float inv_s = sigma > 0.0f ? 1.0f / sigma : 0.0f;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) y[c] = t[c] * inv_s;
+    // w = G_K y  (= B v');  n^2 = y . w (= ||v'||^2);  z = w / n (= B v)
+#pragma unroll
+    for (int rr = 0; rr < RPW; ++rr) {
+      float acc = 0.0f;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) acc = fmaf(gk[rr][c], y[c], acc);
+      part[rr] = acc;
+    }
+    red = warp_transpose_reduce<RPW>(part, lane, idx);
+    if (transpose_reduce_writer<RPW>(lane)) ws[warp * RPW + idx] = red;
+    __syncthreads();
+    float wv[CPL], n2 = 0.0f;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) {
+      wv[c] = ws[lane * CPL + c];
+      n2 = fmaf(y[c], wv[c], n2);
+    }
+    n2 = fmaxf(warp_sum(n2), 0.0f);
+    const float n = sqrtf(n2);
+    inv_n = n > 0.0f ? 1.0f / n : 0.0f;
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) z[c] = wv[c] * inv_n;
+  }
+  if (warp == 0) {
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) a.ybuf[hidx * DH + lane * CPL + c] = y[c] * inv_n;
+  }
+  if (tid == 0) {
+    a.sigma[hidx] = sigma;
+    if (!isfinite(sigma)) set_status(a.status, GAS_DEV_NONFINITE_SIGMA);
+    if (a.scale_out != nullptr) atomic_max_nonneg(&a.scale_out[l], a.scale_c * sigma);
+  }
+}
+
+template <int NZ>
+cudaError_t launch_gram_nz(const GramArgs& a, int num_sms, cudaStream_t st) {
+  using Cfg = GramCfg<NZ>;
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(gram_kernel<NZ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(Cfg::kSmem));
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  const int T = a.s.L * (a.s.tiles_k + a.s.tiles_q);
+  const int grid = T < num_sms ? T : num_sms;
+  gram_kernel<NZ><<<grid, kGramThreads, Cfg::kSmem, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t gram_smem_bytes(int nz) {
+  switch (nz) {
+    case 16: return GramCfg<16>::kSmem;
+    case 32: return GramCfg<32>::kSmem;
+    case 64: return GramCfg<64>::kSmem;
+    case 128: return GramCfg<128>::kSmem;
+    default: return 0;
+  }
+}
+
+cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st) {
+  prep_v_kernel<<<a.s.L * a.s.nq, 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gram(const GramArgs& a, int num_sms, cudaStream_t st) {
+  switch (a.s.nz) {
+    case 16: return launch_gram_nz<16>(a, num_sms, st);
+    case 32: return launch_gram_nz<32>(a, num_sms, st);
+    case 64: return launch_gram_nz<64>(a, num_sms, st);
+    case 128: return launch_gram_nz<128>(a, num_sms, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st) {
+  if (a.s.dh == 128) iterate_kernel<128><<<a.s.L * a.s.nq, 256, 0, st>>>(a);
+  else if (a.s.dh == 64) iterate_kernel<64><<<a.s.L * a.s.nq, 256, 0, st>>>(a);
+  else return cudaErrorInvalidValue;
+  return cudaGetLastError();
+}
+
+}  // namespace gas

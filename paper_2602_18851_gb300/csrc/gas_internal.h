@@ -1,0 +1,120 @@
+// Internal declarations shared by the host API (gas_api.cpp) and the kernels.
+// Nothing here is part of the public C ABI (include/gas.h).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#ifndef GAS_DEV_NONFINITE_SIGMA
+#define GAS_DEV_NONFINITE_SIGMA 0x1
+#define GAS_DEV_WAIT_TIMEOUT 0x2
+#endif
+
+namespace gas {
+
+constexpr int kMaxLayers = 512;             // per-layer pointer table carried as a kernel parameter
+constexpr int kStreamChunk = 256;           // columns of d per streaming CTA
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // bounded device waits: 2 s
+
+// Per-layer base pointers of the bf16 weight blocks, passed by value.
+struct LayerTable {
+  const uint16_t* q[kMaxLayers];
+  const uint16_t* k[kMaxLayers];
+};
+
+// Shape of one handle.
+struct Shape {
+  int L, d, nq, nkv, dh, G;
+  int nch;        // ceil(d / kStreamChunk)
+  int tiles_q;    // ceil(nq * dh / 128)
+  int tiles_k;    // ceil(nkv * dh / 128)
+  int nkc;        // ceil(d / 64)
+  int nz;         // z-accumulator columns of a K tile (multiple of 16)
+};
+
+// ---- streaming matvec-chain passes (Algorithm 2 applied literally) ---------------
+// One pass streams one weight matrix X (a head's A_h or a group's B_g, d_h x d) in
+// column chunks.  For every vector that uses X it forms p = X^T x over the chunk
+// (and ||p||^2), then either q = X p (partial over the chunk) or writes p out.
+enum StreamMode : int {
+  kPassQ = 0,      // X = A_h, x = z from K partials; out: t = A_h u' partials, ||u'||^2
+  kPassK = 1,      // X = B_g, x = y from Q partials (G heads); out: z = B_g v', ||v'||^2
+  kPassK0 = 2,     // X = B_g, p = v_in chunk (G heads); out: z = B_g v, ||v||^2
+  kPassKOut = 3,   // X = B_g, x = y (G heads); writes p (= v') to v_out, ||v'||^2
+};
+
+struct StreamArgs {
+  Shape s;
+  int mode;
+  int in_nch;         // number of partial chunks to sum for the input vector
+  int in_scaled;      // 1: x = sum(in) / sqrt(sum(in2)); 0: x = sum(in)
+  const float* in;    // [L][nq][in_nch][dh]
+  const float* in2;   // [L][nq][in_nch]
+  float* out;         // [L][nq][nch][dh] (q partials)      (modes Q, K, K0)
+  float* out2;        // [L][nq][nch]     (||p||^2 partials) (all modes)
+  const float* v_in;  // [L][nq][d]                          (mode K0)
+  float* v_out;       // [L][nq][d]                          (mode KOut)
+  float* s_zero;      // mode K0: per-layer scale slots zeroed for the fused epilogue
+};
+
+struct FinalizeArgs {
+  Shape s;
+  const float* s2p;   // [L][nq][nch] ||u'||^2 partials of the last Q pass
+  const float* n2p;   // [L][nq][nch] ||v'||^2 partials of the last K pass (or null)
+  float* v_out;       // [L][nq][d] raw v' (normalised in place) or null
+  float* sigma;       // [L][nq]
+  float* scale_out;   // [L] fused scale (atomic max) or null
+  float scale_c;      // alpha * d / sqrt(d_h) / (eta * r_max)
+  unsigned* status;
+};
+
+// ---- Gram path --------------------------------------------------------------------
+struct PrepArgs {
+  Shape s;
+  const float* v_in;   // [L][nq][d]
+  uint16_t* vhl;       // [L][tiles_k][nz][d] bf16 hi/lo rows of v / ||v||
+  float* s_zero;       // [L] or null
+};
+
+struct GramArgs {
+  Shape s;
+  const CUtensorMap* maps_q;  // [L] tensor maps over Wq[l] ([nq*dh, d], box 64 x 128)
+  const CUtensorMap* maps_k;  // [L]
+  const CUtensorMap* map_v;   // one map over vhl ([L*tiles_k*nz, d], box 64 x nz)
+  float* gq;                  // [L][tiles_q][128][128]
+  float* gk;                  // [L][tiles_k][128][128]
+  float* z0;                  // [L][nq][2][dh] (hi and lo halves of B_g v/||v||)
+  unsigned* status;
+};
+
+struct IterArgs {
+  Shape s;
+  int iters;
+  const float* gq;
+  const float* gk;
+  const float* z0;
+  float* ybuf;        // [L][nq][dh]  y / ||v'|| of the last iteration (write-back input)
+  float* sigma;       // [L][nq]
+  float* scale_out;   // [L] fused scale (atomic max) or null
+  float scale_c;
+  unsigned* status;
+};
+
+struct ScalesArgs {
+  int L, nq;
+  const float* sigma;
+  float* s;
+  float scale_c;
+};
+
+// Launchers (return cudaGetLastError() of the launch).
+cudaError_t launch_stream_pass(const LayerTable& tab, const StreamArgs& a, cudaStream_t st);
+cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st);
+cudaError_t launch_scales(const ScalesArgs& a, cudaStream_t st);
+cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st);
+cudaError_t launch_gram(const GramArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st);
+size_t gram_smem_bytes(int nz);
+
+}  // namespace gas

@@ -1,0 +1,281 @@
+"""GPU parity: the CUDA library against the float64 oracle on the same seeded inputs.
+
+sigma and the per-layer scale must match within 1e-3 relative (at the same iteration
+count and start vectors), v_out within 1e-3 Euclidean distance, and head / group
+indexing exactly (one-hot weights).  Both back ends are covered; small workloads are
+compared on every head, the full Llama-2-70B shape on whole sampled layers.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from synth import get_workload, make_start_vectors
+from tests.parity_utils import (assert_sigma_close, assert_v_close, gpu_inputs, oracle_for,
+                                oracle_scales, run_library)
+
+pytestmark = pytest.mark.gpu
+
+METHODS = ["gram", "stream"]
+SMALL = ["tiny-mha", "tiny-gqa", "tiny-gqa128", "ragged", "ragged128", "gpt2-small"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import paper_2602_18851_gb300 as gas
+    gas.build()
+    gas.load()
+
+
+@pytest.mark.parametrize("method", METHODS)
+@pytest.mark.parametrize("name", SMALL)
+def test_small_workloads_all_heads(name, method):
+    wl = get_workload(name)
+    torch.manual_seed(0)
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    got = run_library(wl, wq, wk, v_in, method=method)
+    sig, v = oracle_for(wl, wq, wk, v_in)
+    assert_sigma_close(got["sigma"].ravel(), sig)
+    assert_v_close(got["v_out"], v)
+    s_ref = oracle_scales(wl, sig.reshape(wl.layers, wl.n_q))
+    assert_sigma_close(got["s"], s_ref, what="scale")
+    assert got["status"] == 0
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_gpt2_xl_all_heads(method):
+    wl = get_workload("gpt2-xl")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    got = run_library(wl, wq, wk, v_in, method=method)
+    sig, v = oracle_for(wl, wq, wk, v_in)
+    assert_sigma_close(got["sigma"].ravel(), sig)
+    assert_v_close(got["v_out"], v)
+    assert_sigma_close(got["s"], oracle_scales(wl, sig.reshape(wl.layers, wl.n_q)), what="scale")
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_llama2_7b_planted_all_heads_and_closed_form(method):
+    wl = get_workload("llama2-7b-planted")
+    wq, wk, v_in, meta = gpu_inputs(wl)
+    got = run_library(wl, wq, wk, v_in, method=method)
+    sig, v = oracle_for(wl, wq, wk, v_in)
+    assert_sigma_close(got["sigma"].ravel(), sig)
+    assert_v_close(got["v_out"], v)
+    # closed form: sigma_1 = s^Q_1 s^K_1 up to the Weyl bound of the bf16 rounding
+    s_true = meta["sigma_planted"].numpy()
+    weyl = (meta["err_q"] * meta["norm_k"] + meta["norm_q"] * meta["err_k"]
+            + meta["err_q"] * meta["err_k"]).numpy()
+    err = np.abs(got["sigma"] - s_true)
+    assert np.all(err <= weyl + 1e-4 * s_true)
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_llama2_70b_gqa_sampled_layers(method):
+    """Full 70B shape (80 layers, d 8192, 64/8 heads, d_h 128, 30 iterations) in the
+    launch configuration the benchmark times; oracle on every head of 3 layers."""
+    wl = get_workload("llama2-70b-gqa")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    got = run_library(wl, wq, wk, v_in, method=method, iters=wl.iters if method == "gram" else 4)
+    iters = wl.iters if method == "gram" else 4
+    layers = [0, 39, 79]
+    pairs = [(l, h) for l in layers for h in range(wl.n_q)]
+    sig, v = oracle_for(wl, wq, wk, v_in, pairs=pairs, iters=iters)
+    gs = np.array([got["sigma"][l, h] for l, h in pairs])
+    gv = np.stack([got["v_out"][l, h] for l, h in pairs])
+    assert_sigma_close(gs, sig)
+    assert_v_close(gv, v)
+    s_ref = oracle_scales(wl, sig.reshape(len(layers), wl.n_q), n_heads_total=wl.layers * wl.n_q)
+    assert_sigma_close(got["s"][layers], s_ref, what="scale")
+    assert np.all(np.isfinite(got["sigma"])) and np.all(got["sigma"] > 0)
+    del wq, wk, v_in
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("method", METHODS)
+@pytest.mark.parametrize("iters", [1, 2, 5])
+def test_iteration_counts(method, iters):
+    wl = get_workload("tiny-gqa128")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    got = run_library(wl, wq, wk, v_in, method=method, iters=iters)
+    sig, v = oracle_for(wl, wq, wk, v_in, iters=iters)
+    assert_sigma_close(got["sigma"].ravel(), sig)
+    assert_v_close(got["v_out"], v)
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_unfused_scales_and_no_writeback(method):
+    wl = get_workload("tiny-gqa")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    a = run_library(wl, wq, wk, v_in, method=method, fused=False, write_back=False)
+    b = run_library(wl, wq, wk, v_in, method=method, fused=True, write_back=True)
+    assert a["v_out"] is None
+    np.testing.assert_array_equal(a["sigma"], b["sigma"])
+    np.testing.assert_allclose(a["s"], b["s"], rtol=1e-6)
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_calibration_options(method):
+    wl = get_workload("tiny-mha")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    sig, _ = oracle_for(wl, wq, wk, v_in)
+    sig = sig.reshape(wl.layers, wl.n_q)
+    for gamma, delta, rmax, ao in [(2.5, 1e-6, 448.0, 0.0), (0.0, 1e-3, 448.0, 0.0),
+                                   (0.0, 1e-6, 57344.0, 0.0), (0.0, 1e-6, 448.0, 0.08)]:
+        got = run_library(wl, wq, wk, v_in, method=method, gamma=gamma, delta=delta, r_max=rmax,
+                          alpha_override=ao)
+        ref = oracle_scales(wl, sig, gamma=gamma, delta=delta, r_max=rmax, alpha_override=ao)
+        assert_sigma_close(got["s"], ref, what="scale")
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_one_hot_group_indexing_exact(method):
+    """Only KV group g non-zero -> exactly the heads h with h // G == g have sigma > 0;
+    only query head h non-zero -> exactly that head has sigma > 0."""
+    import paper_2602_18851_gb300 as gas
+    L, d, nq, nkv, dh = 2, 512, 8, 2, 128
+    gen = torch.Generator(device="cuda").manual_seed(5)
+    wq_full = [torch.randn(nq * dh, d, device="cuda", generator=gen).to(torch.bfloat16) for _ in range(L)]
+    v_in = torch.randn(L, nq, d, device="cuda", generator=gen)
+    with gas.Handle(L, d, nq, nkv, dh) as h:
+        h.set_method(method)
+        for g in range(nkv):
+            wk = []
+            for _ in range(L):
+                w = torch.zeros(nkv * dh, d, device="cuda")
+                w[g * dh:(g + 1) * dh] = torch.randn(dh, d, device="cuda", generator=gen)
+                wk.append(w.to(torch.bfloat16))
+            sigma, _ = h.spectral_norms(wq_full, wk, 3, v_in)
+            nz = (sigma > 0).cpu().numpy()
+            expect = np.zeros((L, nq), dtype=bool)
+            expect[:, g * (nq // nkv):(g + 1) * (nq // nkv)] = True
+            assert np.array_equal(nz, expect)
+        wk_full = [torch.randn(nkv * dh, d, device="cuda", generator=gen).to(torch.bfloat16)
+                   for _ in range(L)]
+        for hq in [0, 3, 7]:
+            wq = []
+            for _ in range(L):
+                w = torch.zeros(nq * dh, d, device="cuda")
+                w[hq * dh:(hq + 1) * dh] = torch.randn(dh, d, device="cuda", generator=gen)
+                wq.append(w.to(torch.bfloat16))
+            sigma, v_out = h.spectral_norms(wq, wk_full, 3, v_in)
+            nz = (sigma > 0).cpu().numpy()
+            expect = np.zeros((L, nq), dtype=bool)
+            expect[:, hq] = True
+            assert np.array_equal(nz, expect)
+            vo = v_out.cpu().numpy()
+            assert np.all(vo[:, [x for x in range(nq) if x != hq]] == 0.0)
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_zero_start_vectors_and_inplace_warm_start(method):
+    import paper_2602_18851_gb300 as gas
+    wl = get_workload("tiny-gqa128")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    v_in[1, 3].zero_()
+    v_in[0, 0].zero_()
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        h.set_method(method)
+        sig_ref, v_ref = oracle_for(wl, wq, wk, v_in, iters=4)
+        v = v_in.clone()
+        sigma, vo = h.spectral_norms(wq, wk, 4, v, v_out=v)  # v_out aliases v_in
+        assert vo.data_ptr() == v.data_ptr()
+        torch.cuda.synchronize()
+        s = sigma.cpu().numpy()
+        assert s[1, 3] == 0.0 and s[0, 0] == 0.0
+        assert np.all(v[1, 3].cpu().numpy() == 0.0)
+        assert_sigma_close(s.ravel(), sig_ref)
+        assert_v_close(v.cpu().numpy(), v_ref)
+        # warm start continues the iteration: 4 + 3 iterations == 7 from the start
+        sigma2, _ = h.spectral_norms(wq, wk, 3, v, v_out=v)
+        sig7, _ = oracle_for(wl, wq, wk, v_in, iters=7)
+        assert_sigma_close(sigma2.cpu().numpy().ravel(), sig7, rtol=2e-3)
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_nonfinite_weights_flag_status(method):
+    import paper_2602_18851_gb300 as gas
+    wl = get_workload("tiny-gqa")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    wq[1][5, 7] = float("nan")
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        h.set_method(method)
+        sigma, s, _ = h.refresh(wq, wk, 3, v_in)
+        torch.cuda.synchronize()
+        st = h.device_status(clear=True)
+        assert st & gas.GAS_DEV_NONFINITE_SIGMA
+        assert torch.isnan(s[1]).item()
+        assert torch.isfinite(s[0]).item()
+        assert torch.isfinite(sigma[0]).all().item()
+        assert h.device_status() == 0
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_deterministic_and_side_stream(method):
+    import paper_2602_18851_gb300 as gas
+    wl = get_workload("tiny-gqa128")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        h.set_method(method)
+        a, sa, va = h.refresh(wq, wk, wl.iters, v_in)
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            b, sb, vb = h.refresh(wq, wk, wl.iters, v_in, stream=side)
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        assert torch.equal(a, b) and torch.equal(sa, sb) and torch.equal(va, vb)
+
+
+def test_methods_agree_with_each_other():
+    wl = get_workload("gpt2-small")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    a = run_library(wl, wq, wk, v_in, method="gram")
+    b = run_library(wl, wq, wk, v_in, method="stream")
+    assert_sigma_close(a["sigma"].ravel(), b["sigma"].ravel(), rtol=1e-4)
+
+
+def test_transient_refresh_tracks_oracle():
+    """Llama-2-70B transient workload, abridged to keep the test short: cold start of
+    30 iterations, then warm-started refreshes of 2 iterations while the weights take a
+    seeded rank-8 step every call (spike of 5e-2 at steps 40-45).  GPU and oracle each
+    carry their own v; sigma and the layer scale are compared on a sampled layer."""
+    from synth.gen import TransientWeights
+    import paper_2602_18851_gb300 as gas
+    import oracle
+    from tests.helpers import tensor_bits
+    wl = get_workload("llama2-70b-transient").scaled(layers=4)
+    tw = TransientWeights(wl, device="cuda")
+    v = make_start_vectors(wl, device="cuda")
+    layer = 2
+    v_or = v[layer:layer + 1].cpu().numpy().copy()
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        for t in range(48):
+            if t > 0:
+                tw.step(t)
+            iters = wl.cold_iters if t == 0 else wl.iters
+            sigma, s, v = h.refresh(tw.wq, tw.wk, iters, v, v_out=v)
+            qb = [tensor_bits(tw.wq[layer])]
+            kb = [tensor_bits(tw.wk[layer])]
+            pairs = [(0, hq) for hq in range(wl.n_q)]
+            sig_o, vv = oracle.heads(wl.d, wl.n_q, wl.n_kv, wl.d_h, qb, kb, v_or, iters, pairs)
+            v_or = vv.reshape(1, wl.n_q, wl.d).astype(np.float32)
+            assert_sigma_close(sigma[layer].cpu().numpy(), sig_o, rtol=1e-3)
+            s_ref = oracle_scales(wl, sig_o.reshape(1, wl.n_q), n_heads_total=wl.layers * wl.n_q)
+            assert_sigma_close(s[layer:layer + 1].cpu().numpy(), s_ref, what="scale")
+
+
+def test_bf16_inputs_unchanged():
+    """The library never writes the weights or v_in (when v_out is separate)."""
+    import paper_2602_18851_gb300 as gas
+    wl = get_workload("tiny-gqa")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    cq = [w.clone() for w in wq]
+    cv = v_in.clone()
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        for m in METHODS:
+            h.set_method(m)
+            h.refresh(wq, wk, 3, v_in)
+    torch.cuda.synchronize()
+    assert all(torch.equal(a, b) for a, b in zip(cq, wq))
+    assert torch.equal(cv, v_in)
+
