@@ -43,6 +43,7 @@ def parse():
     p.add_argument("--workload", default="llama2-70b-gqa")
     p.add_argument("--method", default="auto", choices=["auto", "gram", "stream"])
     p.add_argument("--iters", type=int, default=0, help="override the workload's iteration count")
+    p.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling case)")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU-baseline sample budget")
@@ -197,6 +198,8 @@ def run_reference(args, rank, world):
     if rank != 0:
         return
     wl = get_workload(args.workload)
+    if args.layers:
+        wl = wl.scaled(layers=args.layers)
     iters = args.iters or wl.iters
     steps, warm = max(1, args.steps), max(0, args.warmup)
     budget = max(0.5, min(6.0, 150.0 / max(1, steps + warm)))
@@ -234,6 +237,8 @@ def main():
     dev = torch.device("cuda", local)
     gas.build()
     wl = get_workload(args.workload)
+    if args.layers:
+        wl = wl.scaled(layers=args.layers)
     iters = args.iters or wl.iters
     wq, wk, _ = make_weights(wl, device=dev)
     v_in = make_start_vectors(wl, device=dev)

@@ -53,7 +53,7 @@ def _status_name(s: int) -> str:
 
 
 def build(force: bool = False) -> str:
-    from .build import build as _build
+    from .builder import build as _build
     return _build(force=force)
 
 
@@ -70,7 +70,7 @@ def load(path: str = LIB_PATH):
     if _lib is not None:
         return _lib
     if not os.path.exists(path):
-        raise OSError(f"{path} not found: build it with python -m paper_2602_18851_gb300.build")
+        raise OSError(f"{path} not found: build it with python -m paper_2602_18851_gb300.builder")
     lib = ctypes.CDLL(path)
     vp, c_int, c_double, c_ll = ctypes.c_void_p, ctypes.c_int, ctypes.c_double, ctypes.c_longlong
     lib.gas_create.argtypes = [c_int] * 5 + [ctypes.POINTER(vp)]

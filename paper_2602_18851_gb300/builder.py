@@ -1,6 +1,6 @@
 """Build ``libgas.so`` in-tree with nvcc for sm_103a (one -gencode, objects in parallel).
 
-    python -m paper_2602_18851_gb300.build [--force]
+    python -m paper_2602_18851_gb300.builder [--force]
 """
 
 import concurrent.futures as cf

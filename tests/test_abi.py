@@ -129,3 +129,15 @@ def test_gpu_workspace_and_resolve(lib):
         assert a == pytest.approx(calib.alpha_min(g, 8192, 128, 5120, 1024, 1e-6), rel=1e-12)
         h.set_calibration(alpha_override=0.02)
         assert h.resolve_calibration()[1] == 0.02
+
+
+def test_graft_entry_build():
+    """__graft_entry__.build() compiles the library (sm_103a) and the oracle and imports."""
+    import importlib
+    import sys
+    import os
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    sys.path.insert(0, root)
+    ge = importlib.import_module("__graft_entry__")
+    ge.build()
+    assert os.path.exists(gas.LIB_PATH)
