@@ -41,7 +41,7 @@ def parse():
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="llama2-70b-gqa")
-    p.add_argument("--method", default="auto", choices=["auto", "gram", "stream"])
+    p.add_argument("--method", default="auto", choices=["auto", "fused", "gram", "stream"])
     p.add_argument("--iters", type=int, default=0, help="override the workload's iteration count")
     p.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling case)")
     p.add_argument("--no-e2e", action="store_true")
@@ -292,11 +292,11 @@ def main():
     weight_b = wl.weight_bytes()
     v_b = 4 * wl.layers * wl.n_q * wl.d
     algo_step = weight_b + 2 * v_b
-    method = names and ("gram" if "gram" in names else "stream")
-    if method == "gram":
-        dom = "gram"
+    method = "fused" if "gram_fused" in names else ("gram" if "gram" in names else "stream")
+    if method in ("fused", "gram"):
+        dom = "gram_fused" if method == "fused" else "gram"
         dom_bytes = weight_b + v_b     # every W^Q_h and W^K_g once + the start vectors
-        dom_ms = kern_ms["gram"]
+        dom_ms = kern_ms[dom]
     else:
         dom = "stream_pass_q"
         n_q_launch = launches.get("stream_pass_q", 1)

@@ -54,9 +54,12 @@ typedef enum {
 #define GAS_DEV_WAIT_TIMEOUT    0x2  /* a bounded mbarrier/flag wait gave up */
 
 /* Power-iteration back ends (gas_set_method). */
-#define GAS_METHOD_AUTO   0  /* library picks (Gram for every iteration count it supports) */
+#define GAS_METHOD_AUTO   0  /* library picks (the fused Gram back end) */
 #define GAS_METHOD_STREAM 1  /* per-iteration streaming matvec chain, Algorithm 2 literally */
-#define GAS_METHOD_GRAM   2  /* one weight pass to d_h x d_h Gram matrices, iterate in R^{d_h} */
+#define GAS_METHOD_GRAM   2  /* one weight pass to d_h x d_h Gram matrices, iterate in R^{d_h}
+                                (separate iteration kernel) */
+#define GAS_METHOD_FUSED  3  /* as GRAM, with the iterations run inside the Gram kernel from
+                                tensor memory (cooperative launch: needs every SM free) */
 
 /*
  * Create a handle for one model shape (the paper's Section 4 cost model

@@ -33,7 +33,8 @@ GAS_DEV_WAIT_TIMEOUT = 0x2
 METHOD_AUTO = 0
 METHOD_STREAM = 1
 METHOD_GRAM = 2
-METHODS = {"auto": METHOD_AUTO, "stream": METHOD_STREAM, "gram": METHOD_GRAM}
+METHOD_FUSED = 3
+METHODS = {"auto": METHOD_AUTO, "stream": METHOD_STREAM, "gram": METHOD_GRAM, "fused": METHOD_FUSED}
 
 E4M3_MAX = 448.0
 
@@ -268,4 +269,4 @@ class Handle:
 
 
 __all__ = ["Handle", "GasError", "load", "build", "gamma_min", "alpha_min", "exported_names",
-           "METHOD_AUTO", "METHOD_STREAM", "METHOD_GRAM", "E4M3_MAX", "LIB_PATH"]
+           "METHOD_AUTO", "METHOD_STREAM", "METHOD_GRAM", "METHOD_FUSED", "E4M3_MAX", "LIB_PATH"]

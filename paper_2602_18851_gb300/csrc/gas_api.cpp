@@ -46,6 +46,8 @@ struct gas_ctx {
   float* z0 = nullptr;
   float* ybuf = nullptr;
   CUtensorMap* dmaps = nullptr;  // [2L + 1]: q maps, k maps, v map
+  unsigned* flags = nullptr;     // [L][tiles_k] key-tile flags of the fused kernel
+  unsigned epoch = 0;            // last flag value used
 
   // host copies of the encoded descriptors and the pointers they were built for
   std::vector<CUtensorMap> hmaps;
@@ -234,7 +236,7 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
 // ---------------- Gram back end ----------------
 gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, const gas::LayerTable& tab,
                     int iters, const float* v_in, float* v_out, float* sigma, float* s_out, float scale_c,
-                    cudaStream_t st) {
+                    bool fused, cudaStream_t st) {
   const Shape& s = h->s;
   gas_status gs = ensure_maps(h, wq, wk, st);
   if (gs != GAS_OK) return gs;
@@ -256,10 +258,20 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
     g.gk = h->gk;
     g.z0 = h->z0;
     g.status = h->status;
-    e = launch(h, "gram", st, [&] { return gas::launch_gram(g, h->num_sms, st); });
+    if (fused) {
+      h->epoch = h->epoch == 0xFFFFFFFFu ? 1u : h->epoch + 1u;
+      g.flags = h->flags;
+      g.epoch = h->epoch;
+      g.iters = iters;
+      g.ybuf = h->ybuf;
+      g.sigma = sigma;
+      g.scale_out = s_out;
+      g.scale_c = scale_c;
+    }
+    e = launch(h, fused ? "gram_fused" : "gram", st, [&] { return gas::launch_gram(g, h->num_sms, fused, st); });
     ++launches;
   }
-  if (e == cudaSuccess) {
+  if (e == cudaSuccess && !fused) {
     gas::IterArgs it{};
     it.s = s;
     it.iters = iters;
@@ -308,9 +320,9 @@ gas_status spectral_impl(gas_ctx* h, const void* const* wq, const void* const* w
   gas::LayerTable tab;
   std::memset(&tab, 0, sizeof(tab));
   fill_table(h, tab, wq, wk);
-  const int method = h->method == GAS_METHOD_AUTO ? GAS_METHOD_GRAM : h->method;
+  const int method = h->method == GAS_METHOD_AUTO ? GAS_METHOD_FUSED : h->method;
   if (method == GAS_METHOD_STREAM) return run_stream(h, tab, iters, v_in, v_out, sigma, s_out, scale_c, st);
-  return run_gram(h, wq, wk, tab, iters, v_in, v_out, sigma, s_out, scale_c, st);
+  return run_gram(h, wq, wk, tab, iters, v_in, v_out, sigma, s_out, scale_c, method == GAS_METHOD_FUSED, st);
 }
 
 gas_status resolve(gas_ctx* h, double gamma, double delta_star, double r_max, double* g_out, double* a_out) {
@@ -392,6 +404,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_z0 = take(L * NQ * 2 * DH * 4);
   const size_t o_y = take(L * NQ * DH * 4);
   const size_t o_maps = take((2 * L + 1) * sizeof(CUtensorMap));
+  const size_t o_flags = take(L * s.tiles_k * sizeof(unsigned));
   h->ws_bytes = off;
   e = cudaMalloc(&h->ws, h->ws_bytes);
   if (e != cudaSuccess) {
@@ -411,6 +424,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   h->z0 = reinterpret_cast<float*>(b + o_z0);
   h->ybuf = reinterpret_cast<float*>(b + o_y);
   h->dmaps = reinterpret_cast<CUtensorMap*>(b + o_maps);
+  h->flags = reinterpret_cast<unsigned*>(b + o_flags);
   h->hmaps.assign(2 * L + 1, CUtensorMap{});
   h->map_q.assign(L, nullptr);
   h->map_k.assign(L, nullptr);
@@ -453,7 +467,8 @@ gas_status gas_set_calibration(gas_handle h, int seq_len, double eta_fp8, double
 
 gas_status gas_set_method(gas_handle h, int method) {
   if (!h) return GAS_ERR_INVALID_ARG;
-  if (method != GAS_METHOD_AUTO && method != GAS_METHOD_STREAM && method != GAS_METHOD_GRAM)
+  if (method != GAS_METHOD_AUTO && method != GAS_METHOD_STREAM && method != GAS_METHOD_GRAM &&
+      method != GAS_METHOD_FUSED)
     return fail(h, GAS_ERR_INVALID_ARG, "unknown method %d", method);
   h->method = method;
   return GAS_OK;

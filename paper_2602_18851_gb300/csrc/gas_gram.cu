@@ -26,7 +26,7 @@ namespace {
 constexpr int kGramThreads = 192;  // warp 0 TMA producer, warp 1 MMA issuer, warps 2-5 epilogue
 constexpr uint32_t kTileBytes = 128u * 64u * 2u;  // one 128-row x 64-column bf16 box
 constexpr int kSmemBudget = 232448;               // 227 KB opt-in dynamic shared memory
-constexpr int kSmemReserve = 2048;                // alignment slack + barriers
+constexpr int kSmemReserve = 4096;                // alignment slack, barriers, epilogue scratch
 
 template <int NZ>
 struct GramCfg {
@@ -99,7 +99,153 @@ __device__ __forceinline__ TileRef decode_tile(const Shape& s, int t) {
   return r;
 }
 
-template <int NZ>
+// Shared scratch of the fused epilogue: per head slot of a tile (two heads per tile
+// when d_h = 64) the current z and y vectors and the per-warp partial dot products.
+struct EpiSmem {
+  float zs[2][128];
+  float ys[2][128];
+  float red[2][2][4];
+  int ok[2];
+};
+
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_u32(unsigned* p, unsigned v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Bounded wait for another CTA's key tile: true once *flag == epoch.
+__device__ bool wait_flag(const unsigned* flag, unsigned epoch, volatile int* abort, unsigned* status) {
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    if (ld_acquire_u32(flag) == epoch) return true;
+    if (*abort) return false;
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      *abort = 1;
+      set_status(status, GAS_DEV_WAIT_TIMEOUT);
+      return false;
+    }
+    __nanosleep(128);
+  }
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+
+// k power iterations for the head(s) of one query tile, in R^{d_h}, with G_Q read from
+// the tile's tensor-memory accumulator and G_K / z0 from the key tile published by
+// (possibly) another CTA.  One thread per row r of the head's d_h x d_h block; the
+// recurrence is the one of iterate_kernel below (Algorithm 2 in R^{d_h}).
+template <int DH>
+__device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int idx, uint32_t tacc, int row,
+                                              int lane, EpiSmem* ep, volatile int* abort) {
+  constexpr int HPT = 128 / DH;  // heads per 128-row tile
+  constexpr int WPH = DH / 32;   // warps per head
+  const Shape& s = a.s;
+  const int hs = row / DH, r = row % DH, wih = r / 32;
+  const int head = idx * HPT + hs;
+  if (head >= s.nq) return;  // whole warps: a ragged last tile has an empty head slot
+  const int bar = 1 + hs;
+  const int g = head / s.G;
+  const int tk = (g * DH) / 128, og = (g * DH) % 128;
+  const unsigned* flag = a.flags + layer * s.tiles_k + tk;
+  if (r == 0) ep->ok[hs] = wait_flag(flag, a.epoch, abort, a.status) ? 1 : 0;
+  named_bar_sync(bar, DH);
+  if (!ep->ok[hs]) return;
+  (void)ld_acquire_u32(flag);
+  const float* GK = a.gk + static_cast<size_t>(layer * s.tiles_k + tk) * 16384u + og * 128 + og;
+  float gk[DH];  // row r of G_K (stored transposed: element (j, r) is G_K[r][j])
+#pragma unroll
+  for (int j = 0; j < DH; ++j) gk[j] = __ldcg(GK + j * 128 + r);
+  const size_t hidx = static_cast<size_t>(layer) * s.nq + head;
+  float z = __ldcg(a.z0 + (hidx * 2) * DH + r) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + r);
+  float* zs = ep->zs[hs];
+  float* ys = ep->ys[hs];
+  zs[r] = z;
+  named_bar_sync(bar, DH);
+  const uint32_t tq = tacc + static_cast<uint32_t>(hs * DH);
+  float sigma = 0.0f, inv_n = 0.0f, y = 0.0f;
+  for (int it = 0; it < a.iters; ++it) {
+    // t = G_Q z (row r);  sigma^2 = z . t;  y = t / sigma
+    float t0 = 0.0f, t1 = 0.0f, t2 = 0.0f, t3 = 0.0f;
+#pragma unroll
+    for (int c0 = 0; c0 < DH; c0 += 32) {
+      uint32_t v[32];
+      tmem_ld32(tq + c0, v);
+      tmem_ld_wait();
+#pragma unroll
+      for (int jj = 0; jj < 32; jj += 4) {
+        const float4 zz = *reinterpret_cast<const float4*>(zs + c0 + jj);
+        t0 = fmaf(__uint_as_float(v[jj + 0]), zz.x, t0);
+        t1 = fmaf(__uint_as_float(v[jj + 1]), zz.y, t1);
+        t2 = fmaf(__uint_as_float(v[jj + 2]), zz.z, t2);
+        t3 = fmaf(__uint_as_float(v[jj + 3]), zz.w, t3);
+      }
+    }
+    const float t = (t0 + t1) + (t2 + t3);
+    float p = warp_sum(z * t);
+    if (lane == 0) ep->red[hs][0][wih] = p;
+    named_bar_sync(bar, DH);
+    float s2 = 0.0f;
+#pragma unroll
+    for (int w = 0; w < WPH; ++w) s2 += ep->red[hs][0][w];
+    s2 = s2 < 0.0f ? 0.0f : s2;
+    sigma = sqrtf(s2);
+    const float inv_s = sigma > 0.0f ? 1.0f / sigma : 0.0f;
+    y = t * inv_s;
+    ys[r] = y;
+    named_bar_sync(bar, DH);
+    // w = G_K y (row r);  n^2 = y . w;  z = w / n
+    float w0 = 0.0f, w1 = 0.0f, w2 = 0.0f, w3 = 0.0f;
+#pragma unroll
+    for (int j = 0; j < DH; j += 4) {
+      const float4 yy = *reinterpret_cast<const float4*>(ys + j);
+      w0 = fmaf(gk[j + 0], yy.x, w0);
+      w1 = fmaf(gk[j + 1], yy.y, w1);
+      w2 = fmaf(gk[j + 2], yy.z, w2);
+      w3 = fmaf(gk[j + 3], yy.w, w3);
+    }
+    const float w = (w0 + w1) + (w2 + w3);
+    p = warp_sum(y * w);
+    if (lane == 0) ep->red[hs][1][wih] = p;
+    named_bar_sync(bar, DH);
+    float n2 = 0.0f;
+#pragma unroll
+    for (int ww = 0; ww < WPH; ++ww) n2 += ep->red[hs][1][ww];
+    n2 = n2 < 0.0f ? 0.0f : n2;
+    const float n = sqrtf(n2);
+    inv_n = n > 0.0f ? 1.0f / n : 0.0f;
+    z = w * inv_n;
+    zs[r] = z;
+    named_bar_sync(bar, DH);
+  }
+  a.ybuf[hidx * DH + r] = y * inv_n;
+  if (r == 0) {
+    a.sigma[hidx] = sigma;
+    if (!isfinite(sigma)) set_status(a.status, GAS_DEV_NONFINITE_SIGMA);
+    if (a.scale_out != nullptr) atomic_max_nonneg(&a.scale_out[layer], a.scale_c * sigma);
+  }
+}
+
+template <int NZ, int DH, bool FUSED>
 __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_constant__ GramArgs a) {
   using Cfg = GramCfg<NZ>;
   constexpr int S = Cfg::kStages;
@@ -114,6 +260,7 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
   uint64_t* done = acce + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  EpiSmem* ep = reinterpret_cast<EpiSmem*>(reinterpret_cast<uint8_t*>(done) + 64);
   volatile int no_abort_flag = 0;
 
   const Shape& s = a.s;
@@ -220,6 +367,13 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
       __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the per-lane wait
       if (!__all_sync(0xFFFFFFFFu, got)) break;
       tc_fence_after();
+      if (FUSED && !tr.is_k) {
+        fused_iterate<DH>(a, tr.layer, tr.idx, tmem + lane_off + acc * 128u, row, lane, ep, abort);
+        tc_fence_before();
+        mbar_arrive(smem_u32(&acce[acc]));
+        ++tc;
+        continue;
+      }
       float* Gout = (tr.is_k ? a.gk : a.gq) +
                     (static_cast<size_t>(tr.layer) * (tr.is_k ? s.tiles_k : s.tiles_q) + tr.idx) * 16384u;
 #pragma unroll 1
@@ -249,6 +403,11 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
                   __uint_as_float(r[jj]);
             }
           }
+        }
+        if (FUSED) {  // publish G_K and z0 of this key tile to the query tiles' epilogues
+          __threadfence();
+          named_bar_sync(3, 128);
+          if (row == 0) st_release_u32(a.flags + tr.layer * s.tiles_k + tr.idx, a.epoch);
         }
       }
       tc_fence_before();
@@ -319,7 +478,8 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
       t[c] = ts[lane * CPL + c];
       s2 = fmaf(z[c], t[c], s2);
     }
-    s2 = fmaxf(warp_sum(s2), 0.0f);
+    s2 = warp_sum(s2);
+    s2 = s2 < 0.0f ? 0.0f : s2;  // rounding can dip below 0; NaN must survive
     sigma = sqrtf(s2);
     const float inv_s = sigma > 0.0f ? 1.0f / sigma : 0.0f;
 #pragma unroll
@@ -341,7 +501,8 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
       wv[c] = ws[lane * CPL + c];
       n2 = fmaf(y[c], wv[c], n2);
     }
-    n2 = fmaxf(warp_sum(n2), 0.0f);
+    n2 = warp_sum(n2);
+    n2 = n2 < 0.0f ? 0.0f : n2;
     const float n = sqrtf(n2);
     inv_n = n > 0.0f ? 1.0f / n : 0.0f;
 #pragma unroll
@@ -358,20 +519,39 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
   }
 }
 
-template <int NZ>
-cudaError_t launch_gram_nz(const GramArgs& a, int num_sms, cudaStream_t st) {
+template <int NZ, int DH, bool FUSED>
+cudaError_t launch_gram_cfg(const GramArgs& a, int num_sms, cudaStream_t st) {
   using Cfg = GramCfg<NZ>;
+  auto kern = gram_kernel<NZ, DH, FUSED>;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(gram_kernel<NZ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(Cfg::kSmem));
     if (e != cudaSuccess) return e;
     configured = true;
   }
   const int T = a.s.L * (a.s.tiles_k + a.s.tiles_q);
   const int grid = T < num_sms ? T : num_sms;
-  gram_kernel<NZ><<<grid, kGramThreads, Cfg::kSmem, st>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kGramThreads);
+  cfg.dynamicSmemBytes = Cfg::kSmem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;  // all CTAs co-resident: key-tile flags cannot deadlock
+  attr[0].val.cooperative = FUSED ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+template <int NZ>
+cudaError_t launch_gram_nz(const GramArgs& a, int num_sms, bool fused, cudaStream_t st) {
+  if (a.s.dh == 128)
+    return fused ? launch_gram_cfg<NZ, 128, true>(a, num_sms, st) : launch_gram_cfg<NZ, 128, false>(a, num_sms, st);
+  if (a.s.dh == 64)
+    return fused ? launch_gram_cfg<NZ, 64, true>(a, num_sms, st) : launch_gram_cfg<NZ, 64, false>(a, num_sms, st);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace
@@ -391,12 +571,12 @@ cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_gram(const GramArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_gram(const GramArgs& a, int num_sms, bool fused, cudaStream_t st) {
   switch (a.s.nz) {
-    case 16: return launch_gram_nz<16>(a, num_sms, st);
-    case 32: return launch_gram_nz<32>(a, num_sms, st);
-    case 64: return launch_gram_nz<64>(a, num_sms, st);
-    case 128: return launch_gram_nz<128>(a, num_sms, st);
+    case 16: return launch_gram_nz<16>(a, num_sms, fused, st);
+    case 32: return launch_gram_nz<32>(a, num_sms, fused, st);
+    case 64: return launch_gram_nz<64>(a, num_sms, fused, st);
+    case 128: return launch_gram_nz<128>(a, num_sms, fused, st);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -82,10 +82,18 @@ struct GramArgs {
   const CUtensorMap* maps_q;  // [L] tensor maps over Wq[l] ([nq*dh, d], box 64 x 128)
   const CUtensorMap* maps_k;  // [L]
   const CUtensorMap* map_v;   // one map over vhl ([L*tiles_k*nz, d], box 64 x nz)
-  float* gq;                  // [L][tiles_q][128][128]
+  float* gq;                  // [L][tiles_q][128][128] (unfused only)
   float* gk;                  // [L][tiles_k][128][128]
   float* z0;                  // [L][nq][2][dh] (hi and lo halves of B_g v/||v||)
   unsigned* status;
+  // fused variant: k iterations in the epilogue, straight from tensor memory
+  unsigned* flags;            // [L][tiles_k] key-tile publication flags (== epoch when ready)
+  unsigned epoch;             // this launch's flag value (never 0)
+  int iters;
+  float* ybuf;                // [L][nq][dh]
+  float* sigma;               // [L][nq]
+  float* scale_out;           // [L] or null
+  float scale_c;
 };
 
 struct IterArgs {
@@ -113,7 +121,7 @@ cudaError_t launch_stream_pass(const LayerTable& tab, const StreamArgs& a, cudaS
 cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st);
 cudaError_t launch_scales(const ScalesArgs& a, cudaStream_t st);
 cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st);
-cudaError_t launch_gram(const GramArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_gram(const GramArgs& a, int num_sms, bool fused, cudaStream_t st);
 cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st);
 size_t gram_smem_bytes(int nz);
 

@@ -16,7 +16,7 @@ from tests.parity_utils import (assert_sigma_close, assert_v_close, gpu_inputs, 
 
 pytestmark = pytest.mark.gpu
 
-METHODS = ["gram", "stream"]
+METHODS = ["fused", "gram", "stream"]
 SMALL = ["tiny-mha", "tiny-gqa", "tiny-gqa128", "ragged", "ragged128", "gpt2-small"]
 
 
@@ -75,8 +75,8 @@ def test_llama2_70b_gqa_sampled_layers(method):
     launch configuration the benchmark times; oracle on every head of 3 layers."""
     wl = get_workload("llama2-70b-gqa")
     wq, wk, v_in, _ = gpu_inputs(wl)
-    got = run_library(wl, wq, wk, v_in, method=method, iters=wl.iters if method == "gram" else 4)
-    iters = wl.iters if method == "gram" else 4
+    iters = 4 if method == "stream" else wl.iters
+    got = run_library(wl, wq, wk, v_in, method=method, iters=iters)
     layers = [0, 39, 79]
     pairs = [(l, h) for l in layers for h in range(wl.n_q)]
     sig, v = oracle_for(wl, wq, wk, v_in, pairs=pairs, iters=iters)
@@ -231,7 +231,10 @@ def test_methods_agree_with_each_other():
     wq, wk, v_in, _ = gpu_inputs(wl)
     a = run_library(wl, wq, wk, v_in, method="gram")
     b = run_library(wl, wq, wk, v_in, method="stream")
+    c = run_library(wl, wq, wk, v_in, method="fused")
     assert_sigma_close(a["sigma"].ravel(), b["sigma"].ravel(), rtol=1e-4)
+    # the fused kernel runs the same fp32 recurrence as the separate iteration kernel
+    assert_sigma_close(c["sigma"].ravel(), a["sigma"].ravel(), rtol=1e-5)
 
 
 def test_transient_refresh_tracks_oracle():
