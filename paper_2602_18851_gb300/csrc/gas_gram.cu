@@ -112,6 +112,20 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// Named barrier with an AND vote: every participating thread gets the AND of `v`.
+__device__ __forceinline__ bool named_bar_and(int id, int nthreads, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(v)), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
 __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
   unsigned v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -365,7 +379,9 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
       const uint32_t acc = tc & 1u, aph = (tc >> 1) & 1u;
       const bool got = mbar_wait(smem_u32(&accf[acc]), aph, abort, a.status);
       __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the per-lane wait
-      if (!__all_sync(0xFFFFFFFFu, got)) break;
+      // One decision for all four epilogue warps, so none of them can be left alone at
+      // a named barrier further down when another gave up.
+      if (!named_bar_and(4, 128, got)) break;
       tc_fence_after();
       if (FUSED && !tr.is_k) {
         fused_iterate<DH>(a, tr.layer, tr.idx, tmem + lane_off + acc * 128u, row, lane, ep, abort);
