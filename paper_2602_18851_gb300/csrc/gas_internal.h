@@ -96,6 +96,15 @@ struct GramArgs {
   float scale_c;
 };
 
+// Tensor-core write-back v_out = B_g^T (y / ||v'||) for every head (group size <= 16).
+struct WbArgs {
+  Shape s;
+  const CUtensorMap* maps_k;  // [L] (box 64 x 128, as for the Gram pass)
+  const float* ybuf;          // [L][nq][dh]
+  float* v_out;               // [L][nq][d]
+  unsigned* status;
+};
+
 struct IterArgs {
   Shape s;
   int iters;
@@ -123,6 +132,8 @@ cudaError_t launch_scales(const ScalesArgs& a, cudaStream_t st);
 cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st);
 cudaError_t launch_gram(const GramArgs& a, int num_sms, bool fused, cudaStream_t st);
 cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st);
+cudaError_t launch_writeback(const WbArgs& a, int num_sms, cudaStream_t st);
 size_t gram_smem_bytes(int nz);
+constexpr int kWbMaxGroup = 16;  // tensor-core write-back handles n_q/n_kv <= 16
 
 }  // namespace gas
