@@ -47,13 +47,16 @@ def _unit_rows(n: int, m: int, gen, device, dtype) -> torch.Tensor:
 
 
 def _orthonormal(batch: int, rows: int, cols: int, gen, device, dtype) -> torch.Tensor:
-    """[batch, rows, cols] with orthonormal columns (QR of a Gaussian matrix)."""
-    x = torch.randn(batch, rows, cols, generator=gen, device=device, dtype=dtype)
+    """[batch, rows, cols] with orthonormal columns (QR of a Gaussian matrix).
+
+    The Gaussian is drawn on `device`; the QR runs on the host (LAPACK), which keeps
+    the draw independent of the device linear-algebra libraries being loadable."""
+    x = torch.randn(batch, rows, cols, generator=gen, device=device, dtype=dtype).cpu()
     q, r = torch.linalg.qr(x)
     # Fix the sign ambiguity of QR so the draw is a function of the seed only.
     sgn = torch.sign(torch.diagonal(r, dim1=-2, dim2=-1))
     sgn[sgn == 0] = 1
-    return q * sgn.unsqueeze(-2)
+    return (q * sgn.unsqueeze(-2)).to(device)
 
 
 def _draw_layer(wl: Workload, layer: int, device, seed: int):
