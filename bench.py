@@ -142,6 +142,30 @@ class ClockSampler:
                 "power_w_max": max(power), "samples": len(sm), "reasons": sorted(reasons)}
 
 
+def profiled_traffic(kernel, layers):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, scaled from the
+    profiled 4-layer slice to `layers` (traffic grows in proportion to the layers).
+    None when the kernel source changed since the counters were taken."""
+    import hashlib
+    import re
+    files = {"gram_fused": ("gram_fused_llama2-70b-gqa-4layers.md", ["gas_gram.cu", "gas_device.cuh"])}
+    if kernel not in files:
+        return None
+    name, srcs = files[kernel]
+    try:
+        text = open(os.path.join(ROOT, "profiles", name)).read()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_layer=(\d+) source_sha1=(\w+) device_sha1=(\w+)", text)
+    if not m:
+        return None
+    csrc = os.path.join(ROOT, "paper_2602_18851_gb300", "csrc")
+    shas = [hashlib.sha1(open(os.path.join(csrc, f), "rb").read()).hexdigest() for f in srcs]
+    if shas != [m.group(2), m.group(3)]:
+        return None
+    return int(m.group(1)) * layers
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -360,7 +384,8 @@ def main():
             "step_achieved_gbs": step_gbs, "algorithmic_bytes_per_step": algo_step,
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
-                         "traffic": None, "algorithmic_bytes": dom_bytes, "kernel_ms": dom_ms},
+                         "traffic": profiled_traffic(dom, wl.layers) if wl.d == 8192 else None,
+                         "algorithmic_bytes": dom_bytes, "kernel_ms": dom_ms},
             "kernels_ms_per_step": kern_ms,
             "gpu_launches": nl * K,
             "launches_per_step": nl,
