@@ -165,6 +165,34 @@ gas_status gas_set_launch_events(gas_handle h, void *const *events, int n_events
 /* Kernel name of launch i of the last call ("" when out of range). */
 const char *gas_last_launch_name(gas_handle h, int i);
 
+/*
+ * Allocation-free spectral norms (no counterpart in the paper).
+ *
+ * For callers that cannot allocate device memory: code running under another
+ * framework's memory manager that owns all of HBM, latency-critical paths where the
+ * device synchronisation implied by cudaMalloc / cudaFree is not allowed, and plugins
+ * with nowhere to keep a handle alive.  Same result as gas_spectral_norms with
+ * GAS_METHOD_STREAM (Algorithm 2 per head, streaming matvec chain), but it takes the
+ * shape directly, needs no handle, and calls no cudaMalloc, cudaFree or allocating
+ * library routine: its scratch is a file-scope device array of
+ * GAS_STATIC_SCRATCH_BYTES that every GPU loading the library holds until the
+ * process exits.
+ *   Arguments: as gas_create's shape plus gas_spectral_norms' buffers (wq, wk host
+ *   arrays of device pointers; v_in, v_out, sigma device fp32; v_out may be NULL or
+ *   alias v_in).  Scratch needed: 2*align256(layers*n_q*ceil(d/256)*d_h*4) +
+ *   2*align256(layers*n_q*ceil(d/256)*4) bytes (e.g. 16.8 MB for 32 layers, d 4096,
+ *   32 heads, d_h 128); larger shapes are rejected with GAS_ERR_UNSUPPORTED.
+ *   Errors: as gas_spectral_norms; gas_last_error(NULL) holds the message.
+ * The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress) and caches it; make that first call before any stream
+ * capture.  All calls share the array and it keeps the last call's contents: calls
+ * whose kernels overlap on the GPU (other streams, other threads) race on it.
+ */
+#define GAS_STATIC_SCRATCH_BYTES (32u * 1024u * 1024u)
+gas_status gas_spectral_norms_static(int layers, int d, int n_q, int n_kv, int d_h,
+                                     const void *const *wq, const void *const *wk, int iters,
+                                     const float *v_in, float *v_out, float *sigma, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -98,6 +98,7 @@ def load(path: str = LIB_PATH):
     lib.gas_set_launch_events.argtypes = [vp, vp, c_int]
     lib.gas_last_launch_name.argtypes = [vp, c_int]
     lib.gas_last_launch_name.restype = ctypes.c_char_p
+    lib.gas_spectral_norms_static.argtypes = [c_int] * 5 + [vp, vp, c_int, vp, vp, vp, vp]
     _lib = lib
     return lib
 

@@ -351,6 +351,8 @@ gas_status resolve(gas_ctx* h, double gamma, double delta_star, double r_max, do
 
 }  // namespace
 
+void gas::set_global_error(const char* msg) { g_create_err = msg; }
+
 extern "C" {
 
 gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle* out) {

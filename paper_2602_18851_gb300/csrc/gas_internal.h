@@ -133,6 +133,7 @@ cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st);
 cudaError_t launch_gram(const GramArgs& a, int num_sms, bool fused, cudaStream_t st);
 cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st);
 cudaError_t launch_writeback(const WbArgs& a, int num_sms, cudaStream_t st);
+void set_global_error(const char* msg);  // message returned by gas_last_error(NULL)
 size_t gram_smem_bytes(int nz);
 constexpr int kWbMaxGroup = 16;  // tensor-core write-back handles n_q/n_kv <= 16
 

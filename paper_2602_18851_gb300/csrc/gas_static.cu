@@ -1,0 +1,163 @@
+// Allocation-free spectral norms: gas_spectral_norms_static (include/gas.h).
+//
+// Some callers of this library cannot allocate device memory at all: code that runs
+// under another framework's memory manager (which owns every byte of HBM and hands
+// out nothing extra), code on a latency-critical path where the implicit device
+// synchronisation of cudaMalloc / cudaFree is not allowed, and small plugins that
+// have no place to keep a handle (and its workspace) alive between calls.  For them
+// this entry point runs the streaming power iteration (the same kernels as
+// GAS_METHOD_STREAM) with its scratch in one file-scope device array instead of a
+// handle's workspace.  The caller still passes every input and output buffer.
+//
+// The array is part of the library's device image: every GPU that loads the library
+// holds kStaticScratchBytes for it until the process exits.  All calls share it, so
+// calls whose kernels overlap on the GPU (two streams, two host threads) race on it.
+
+#include <atomic>
+#include <cstdio>
+#include <cstring>
+
+#include "../../include/gas.h"
+#include "gas_device.cuh"
+
+namespace gas {
+namespace {
+
+constexpr size_t kStaticScratchBytes = GAS_STATIC_SCRATCH_BYTES;
+constexpr int kMaxDevices = 64;
+
+// Host code must not use this name as a device address (see static_scratch_ptr).
+__device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+std::atomic<void*> g_scratch_ptr[kMaxDevices];
+
+size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+
+// Device address of the scratch array on the current device, looked up once per device
+// (the first call on a device does this; it should come before any stream capture).
+cudaError_t static_scratch_ptr(int dev, void** out) {
+  void* p = g_scratch_ptr[dev].load(std::memory_order_acquire);
+  if (p == nullptr) {
+    cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_ptr[dev].store(p, std::memory_order_release);
+  }
+  *out = p;
+  return cudaSuccess;
+}
+
+}  // namespace
+}  // namespace gas
+
+namespace {
+// Errors are reported like gas_create's: gas_last_error(NULL) returns the message.
+gas_status static_fail(gas_status st, const char* msg) {
+  gas::set_global_error(msg);
+  return st;
+}
+
+bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+}  // namespace
+
+extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int n_kv, int d_h,
+                                                const void* const* wq, const void* const* wk, int iters,
+                                                const float* v_in, float* v_out, float* sigma, void* stream) {
+  char buf[256];
+  if (layers < 1 || d < 8 || n_q < 1 || n_kv < 1 || iters < 1)
+    return static_fail(GAS_ERR_INVALID_ARG, "gas_spectral_norms_static: sizes and iters must be positive");
+  if (layers > gas::kMaxLayers || d % 8 != 0 || n_q % n_kv != 0 || (d_h != 64 && d_h != 128))
+    return static_fail(GAS_ERR_UNSUPPORTED,
+                       "gas_spectral_norms_static: needs layers <= 512, d % 8 == 0, n_q % n_kv == 0, d_h 64/128");
+  if (!wq || !wk || !v_in || !sigma)
+    return static_fail(GAS_ERR_INVALID_ARG, "gas_spectral_norms_static: NULL argument");
+  if (!al16(v_in) || (v_out && !al16(v_out)))
+    return static_fail(GAS_ERR_INVALID_ARG, "gas_spectral_norms_static: vectors must be 16-byte aligned");
+  for (int l = 0; l < layers; ++l)
+    if (!wq[l] || !wk[l] || !al16(wq[l]) || !al16(wk[l]))
+      return static_fail(GAS_ERR_INVALID_ARG, "gas_spectral_norms_static: NULL or misaligned weight pointer");
+
+  gas::Shape s{};
+  s.L = layers; s.d = d; s.nq = n_q; s.nkv = n_kv; s.dh = d_h; s.G = n_q / n_kv;
+  s.nch = (d + gas::kStreamChunk - 1) / gas::kStreamChunk;
+  // Scratch: z and t partials [L][n_q][nch][d_h], their squared-norm partials [L][n_q][nch].
+  const size_t vec = static_cast<size_t>(layers) * n_q * s.nch * d_h * sizeof(float);
+  const size_t nrm = static_cast<size_t>(layers) * n_q * s.nch * sizeof(float);
+  const size_t need = 2 * gas::align256(vec) + 2 * gas::align256(nrm);
+  if (need > gas::kStaticScratchBytes) {
+    snprintf(buf, sizeof(buf),
+             "gas_spectral_norms_static: this shape needs %zu bytes of scratch, the static array holds %zu",
+             need, gas::kStaticScratchBytes);
+    return static_fail(GAS_ERR_UNSUPPORTED, buf);
+  }
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= gas::kMaxDevices)
+    return static_fail(GAS_ERR_CUDA, "gas_spectral_norms_static: no usable current device");
+  void* base = nullptr;
+  e = gas::static_scratch_ptr(dev, &base);
+  if (e != cudaSuccess) {
+    snprintf(buf, sizeof(buf), "gas_spectral_norms_static: cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
+    return static_fail(GAS_ERR_CUDA, buf);
+  }
+  char* b = static_cast<char*>(base);
+  float* zp = reinterpret_cast<float*>(b);
+  float* tp = reinterpret_cast<float*>(b + gas::align256(vec));
+  float* n2p = reinterpret_cast<float*>(b + 2 * gas::align256(vec));
+  float* s2p = reinterpret_cast<float*>(b + 2 * gas::align256(vec) + gas::align256(nrm));
+  // Every scratch element a pass reads was written earlier in the same call (each pass
+  // covers all heads, chunks and rows), so nothing has to be cleared between calls.
+
+  gas::LayerTable tab;
+  std::memset(&tab, 0, sizeof(tab));
+  for (int l = 0; l < layers; ++l) {
+    tab.q[l] = static_cast<const uint16_t*>(wq[l]);
+    tab.k[l] = static_cast<const uint16_t*>(wk[l]);
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  gas::StreamArgs a{};
+  a.s = s;
+  a.mode = gas::kPassK0;
+  a.out = zp;
+  a.out2 = n2p;
+  a.v_in = v_in;
+  e = gas::launch_stream_pass(tab, a, st);
+  for (int it = 0; it < iters && e == cudaSuccess; ++it) {
+    gas::StreamArgs q{};
+    q.s = s;
+    q.mode = gas::kPassQ;
+    q.in_nch = s.nch;
+    q.in_scaled = 1;
+    q.in = zp;
+    q.in2 = n2p;
+    q.out = tp;
+    q.out2 = s2p;
+    e = gas::launch_stream_pass(tab, q, st);
+    const bool last = (it == iters - 1);
+    if (e != cudaSuccess || (last && v_out == nullptr)) break;
+    gas::StreamArgs k{};
+    k.s = s;
+    k.mode = last ? gas::kPassKOut : gas::kPassK;
+    k.in_nch = s.nch;
+    k.in_scaled = 1;
+    k.in = tp;
+    k.in2 = s2p;
+    k.out = zp;
+    k.out2 = n2p;
+    k.v_out = v_out;
+    e = gas::launch_stream_pass(tab, k, st);
+  }
+  if (e == cudaSuccess) {
+    gas::FinalizeArgs f{};
+    f.s = s;
+    f.s2p = s2p;
+    f.n2p = n2p;
+    f.v_out = v_out;
+    f.sigma = sigma;
+    e = gas::launch_finalize(f, st);
+  }
+  if (e != cudaSuccess) {
+    snprintf(buf, sizeof(buf), "gas_spectral_norms_static: launch failed: %s", cudaGetErrorString(e));
+    return static_fail(GAS_ERR_CUDA, buf);
+  }
+  return GAS_OK;
+}
