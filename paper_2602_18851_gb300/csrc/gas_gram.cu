@@ -34,6 +34,10 @@ struct GramCfg {
   static constexpr uint32_t kStageBytes = kTileBytes + kVBytes;
   static constexpr int kStages = (kSmemBudget - kSmemReserve) / static_cast<int>(kStageBytes);
   static constexpr size_t kSmem = static_cast<size_t>(kStages) * kStageBytes + kSmemReserve;
+  // Tensor-memory accumulators (G: 128 columns, z: NZ columns each) cycled over tiles:
+  // three when they fit in the 512 columns, so a query tile's epilogue may run its
+  // iterations for two mainloops before the MMA warp needs its accumulator back.
+  static constexpr int kAcc = (3 * (128 + NZ) <= 512) ? 3 : 2;
   static_assert(kStages >= 3, "ring too shallow");
   static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
 };
@@ -213,9 +217,10 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * SB);
   uint64_t* full = bars;
   uint64_t* empty = bars + S;
+  constexpr int NA = Cfg::kAcc;
   uint64_t* accf = bars + 2 * S;
-  uint64_t* acce = accf + 2;
-  uint64_t* done = acce + 2;
+  uint64_t* acce = accf + NA;
+  uint64_t* done = acce + NA;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
   EpiSmem* ep = reinterpret_cast<EpiSmem*>(reinterpret_cast<uint8_t*>(done) + 64);
@@ -228,7 +233,7 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
       mbar_init(smem_u32(&full[i]), 1);
       mbar_init(smem_u32(&empty[i]), 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < NA; ++i) {
       mbar_init(smem_u32(&accf[i]), 1);
       mbar_init(smem_u32(&acce[i]), 128);
     }
@@ -282,11 +287,11 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
         const TileRef tr = decode_tile(s, t);
-        const uint32_t acc = tc & 1u, aph = (tc >> 1) & 1u;
+        const uint32_t acc = tc % NA, aph = (tc / NA) & 1u;
         if (!mbar_wait(smem_u32(&acce[acc]), aph ^ 1u, abort, a.status)) break;
         tc_fence_after();
         const uint32_t dG = tmem + acc * 128u;
-        const uint32_t dZ = tmem + 256u + acc * static_cast<uint32_t>(NZ);
+        const uint32_t dZ = tmem + NA * 128u + acc * static_cast<uint32_t>(NZ);
         for (int kc = 0; kc < s.nkc; ++kc) {
           const uint32_t st = consumed % S, ph = (consumed / S) & 1u;
           if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
@@ -320,7 +325,7 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
     uint32_t tc = 0;
     for (int t = blockIdx.x; t < T; t += gridDim.x) {
       const TileRef tr = decode_tile(s, t);
-      const uint32_t acc = tc & 1u, aph = (tc >> 1) & 1u;
+      const uint32_t acc = tc % NA, aph = (tc / NA) & 1u;
       const bool got = mbar_wait(smem_u32(&accf[acc]), aph, abort, a.status);
       __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the per-lane wait
       // One decision for all four epilogue warps, so none of them can be left alone at
@@ -351,7 +356,7 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
 #pragma unroll 1
         for (int c0 = 0; c0 < NZ; c0 += 16) {
           uint32_t r[16];
-          tmem_ld16(tmem + lane_off + 256u + acc * static_cast<uint32_t>(NZ) + c0, r);
+          tmem_ld16(tmem + lane_off + NA * 128u + acc * static_cast<uint32_t>(NZ) + c0, r);
           tmem_ld_wait();
 #pragma unroll
           for (int jj = 0; jj < 16; ++jj) {

@@ -8,10 +8,11 @@
 //   D[n][c] = sum_i Y[n][i] * B[i][c],   M = 128 (n), N = 64 (c), K = 128 (i),
 // with A = Y split into bf16 hi and lo rows (about 16 bits of mantissa, K-major, staged
 // in shared memory by the epilogue warps) and B = the TMA box of the weight tile read
-// MN-major (its 64 contiguous columns are the N index).  Row layout of Y: group gi of
-// the tile owns rows 32*gi .. 32*gi+31, head j's hi part in row 32*gi + j and its lo
-// part in row 32*gi + 16 + j, non-zero only in the group's own K range, so the epilogue
-// adds the hi and lo rows with one shuffle inside a warp.  Group size <= 16.
+// MN-major (its 64 contiguous columns are the N index).  Row layout of Y: head j of
+// group gi of the tile is number u = gi*G + j; it goes to TMEM lane quarter u % 4 (so
+// all four epilogue warps drain D), slot m = u / 4: hi part in row 32*(u%4) + m, lo part
+// in row 32*(u%4) + 16 + m, non-zero only in the group's own K range.  The epilogue adds
+// the hi and lo rows with one shuffle inside a warp.  Group size <= 16.
 
 #include "gas_device.cuh"
 
@@ -189,7 +190,8 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           }
           const int k = gi * DH + i0;                 // K index of the 8-element chunk
           const int region = k >> 6, chunk = (k & 63) >> 3;
-          const int rhi = 32 * gi + j, rlo = 32 * gi + 16 + j;
+          const int hu = gi * G + j;                  // head slot u -> quarter u%4, row u/4
+          const int rhi = 32 * (hu & 3) + (hu >> 2), rlo = rhi + 16;
           uint8_t* base = ybase + region * 16384;
           *reinterpret_cast<uint4*>(base + rhi * 128 + ((chunk ^ (rhi & 7)) << 4)) =
               make_uint4(hb[0] | (hb[1] << 16), hb[2] | (hb[3] << 16), hb[4] | (hb[5] << 16), hb[6] | (hb[7] << 16));
@@ -216,7 +218,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
         __syncwarp();
         if (!named_bar_and(4, 128, got)) { ok = false; break; }
         tc_fence_after();
-        if (q < GPT) {
+        if (q < GPT * G) {  // this lane quarter holds at least one head
           uint32_t r0[32], r1[32];
           const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + slot * 64u;
           tmem_ld32(taddr, r0);
@@ -229,10 +231,11 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
             o[c] = hi0 + __shfl_down_sync(0xFFFFFFFFu, hi0, 16);
             o[32 + c] = hi1 + __shfl_down_sync(0xFFFFFFFFu, hi1, 16);
           }
-          const int g = w.tile * GPT + q;
-          if (lane < G && g < s.nkv) {
+          const int hu = 4 * lane + q;  // head slot held by this lane's hi row
+          const int g = w.tile * GPT + hu / G;
+          if (lane < 16 && hu < GPT * G && g < s.nkv) {
             const int col0 = w.c0 + 64 * j;
-            float* dst = a.v_out + (static_cast<size_t>(w.layer) * s.nq + g * G + lane) * s.d + col0;
+            float* dst = a.v_out + (static_cast<size_t>(w.layer) * s.nq + g * G + hu % G) * s.d + col0;
 #pragma unroll
             for (int c = 0; c < 64; c += 4)
               if (col0 + c < s.d) *reinterpret_cast<float4*>(dst + c) = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);

@@ -49,10 +49,18 @@ def _unit_rows(n: int, m: int, gen, device, dtype) -> torch.Tensor:
 def _orthonormal(batch: int, rows: int, cols: int, gen, device, dtype) -> torch.Tensor:
     """[batch, rows, cols] with orthonormal columns (QR of a Gaussian matrix).
 
-    The Gaussian is drawn on `device`; the QR runs on the host (LAPACK), which keeps
-    the draw independent of the device linear-algebra libraries being loadable."""
-    x = torch.randn(batch, rows, cols, generator=gen, device=device, dtype=dtype).cpu()
-    q, r = torch.linalg.qr(x)
+    The Gaussian is drawn on `device`.  Large batches are factored there; small ones,
+    and any batch whose device factorisation is unavailable (the device linear-algebra
+    library cannot always be loaded, e.g. under a profiler), on the host."""
+    x = torch.randn(batch, rows, cols, generator=gen, device=device, dtype=dtype)
+    q = r = None
+    if x.is_cuda and x.numel() >= (1 << 22):
+        try:
+            q, r = torch.linalg.qr(x)
+        except RuntimeError:
+            q = r = None
+    if q is None:
+        q, r = torch.linalg.qr(x.cpu())
     # Fix the sign ambiguity of QR so the draw is a function of the seed only.
     sgn = torch.sign(torch.diagonal(r, dim1=-2, dim2=-1))
     sgn[sgn == 0] = 1
