@@ -287,25 +287,13 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
     ++launches;
   }
   if (e == cudaSuccess && v_out != nullptr) {
-    if (s.G <= gas::kWbMaxGroup) {
-      gas::WbArgs w{};
-      w.s = s;
-      w.maps_k = h->dmaps + s.L;
-      w.ybuf = h->ybuf;
-      w.v_out = v_out;
-      w.status = h->status;
-      e = launch(h, "writeback", st, [&] { return gas::launch_writeback(w, h->num_sms, st); });
-    } else {  // larger groups: the streaming K pass does the same product on CUDA cores
-      gas::StreamArgs k{};
-      k.s = s;
-      k.mode = gas::kPassKOut;
-      k.in_nch = 1;
-      k.in_scaled = 0;
-      k.in = h->ybuf;
-      k.out2 = h->n2p;
-      k.v_out = v_out;
-      e = launch(h, "writeback_cuda_cores", st, [&] { return gas::launch_stream_pass(tab, k, st); });
-    }
+    gas::WbArgs w{};
+    w.s = s;
+    w.maps_k = h->dmaps + s.L;
+    w.ybuf = h->ybuf;
+    w.v_out = v_out;
+    w.status = h->status;
+    e = launch(h, "writeback", st, [&] { return gas::launch_writeback(w, h->num_sms, st); });
     ++launches;
   }
   h->last_launches = launches;

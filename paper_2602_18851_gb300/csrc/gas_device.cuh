@@ -255,6 +255,19 @@ __device__ __forceinline__ uint64_t desc_mnmajor_sw128(uint32_t saddr) {
   return d;
 }
 
+// As desc_mnmajor_sw128 for an operand two swizzle atoms (128 elements) wide along
+// M/N: the second 64-element atom starts `atom_stride` bytes after the first (leading
+// byte offset), e.g. the second of two TMA boxes placed back to back.
+__device__ __forceinline__ uint64_t desc_mnmajor_sw128_2atoms(uint32_t saddr, uint32_t atom_stride) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>((atom_stride >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;
+  d |= static_cast<uint64_t>(1u) << 46;
+  d |= static_cast<uint64_t>(2u) << 61;
+  return d;
+}
+
 // Generic-proxy shared-memory writes become visible to the tensor core (async proxy).
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -267,6 +280,11 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
          | (1u << 10)                              // B format: bf16
          | (static_cast<uint32_t>(N >> 3) << 17)   // N / 8
          | (static_cast<uint32_t>(M >> 4) << 24);  // M / 16
+}
+
+// As idesc_bf16_f32 with A MN-major ("transpose A").
+__host__ __device__ constexpr uint32_t idesc_bf16_f32_amn(int M, int N) {
+  return idesc_bf16_f32(M, N) | (1u << 15);
 }
 
 // As idesc_bf16_f32 with B MN-major ("transpose B").

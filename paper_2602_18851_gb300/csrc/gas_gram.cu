@@ -23,10 +23,16 @@ namespace gas {
 
 namespace {
 
-constexpr int kGramThreads = 192;  // warp 0 TMA producer, warp 1 MMA issuer, warps 2-5 epilogue
+// Warp 0: TMA producer; warp 1: MMA issuer (+ TMEM allocation); the rest: epilogue
+// (4 warps for the Gram-only kernel, 8 for the fused one: two threads per row).
+template <bool FUSED>
+struct GramWarps {
+  static constexpr int kEpiWarps = FUSED ? 8 : 4;
+  static constexpr int kThreads = 64 + 32 * kEpiWarps;
+};
 constexpr uint32_t kTileBytes = 128u * 64u * 2u;  // one 128-row x 64-column bf16 box
 constexpr int kSmemBudget = 232448;               // 227 KB opt-in dynamic shared memory
-constexpr int kSmemReserve = 4096;                // alignment slack, barriers, epilogue scratch
+constexpr int kSmemReserve = 6144;                // alignment slack, barriers, epilogue scratch
 
 template <int NZ>
 struct GramCfg {
@@ -103,104 +109,122 @@ __device__ __forceinline__ TileRef decode_tile(const Shape& s, int t) {
   return r;
 }
 
-// Shared scratch of the fused epilogue: per head slot of a tile (two heads per tile
-// when d_h = 64) the current z and y vectors and the per-warp partial dot products.
+// Shared scratch of the fused epilogue, per head slot of a tile (two heads per tile
+// when d_h = 64): the half-row partial sums of t' = G_Q x and of w = G_K y written by
+// the two thread halves, and the per-warp partial dot products.
 struct EpiSmem {
-  float zs[2][128];
-  float ys[2][128];
-  float red[2][2][4];
+  float tsh[2][2][128];  // [slot][half][row]
+  float wsh[2][2][128];
+  float red[2][2][8];    // [slot][which dot][warp of the head group]
   int ok[2];
 };
 
-// k power iterations for the head(s) of one query tile, in R^{d_h}, with G_Q read from
-// the tile's tensor-memory accumulator and G_K / z0 from the key tile published by
-// (possibly) another CTA.  One thread per row r of the head's d_h x d_h block; the
-// recurrence is the one of iterate_kernel below (Algorithm 2 in R^{d_h}).
+// k power iterations for the head(s) of one query tile in R^{d_h}.  Each row r of the
+// head's d_h x d_h block is held by two threads (half = 0, 1), each with half of the
+// row of G_Q (read once from the tile's tensor-memory accumulator, which is then handed
+// back to the MMA warp) and half of the row of G_K (published by the key tile).
+// With x = c z (c a known scalar, c = 1 for z0) one iteration of Algorithm 2 is
+//   t' = G_Q x,  S1 = x.t' = c^2 sigma^2,  y = t' / sqrt(S1),
+//   w  = G_K y,  S2 = y.w = ||v'||^2,       x <- w,  c <- sqrt(S2),
+// so only two barriers per iteration are needed (after t' and after w).
 template <int DH>
 __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int idx, uint32_t tacc, int row,
-                                              int lane, EpiSmem* ep, volatile int* abort) {
-  constexpr int HPT = 128 / DH;  // heads per 128-row tile
-  constexpr int WPH = DH / 32;   // warps per head
+                                              int half, int lane, EpiSmem* ep, volatile int* abort,
+                                              uint32_t acce_bar) {
+  constexpr int HPT = 128 / DH;   // heads per 128-row tile
+  constexpr int HC = DH / 2;      // columns per thread (half a row)
+  constexpr int NT = 2 * DH;      // threads per head
+  constexpr int NW = NT / 32;     // warps per head
   const Shape& s = a.s;
-  const int hs = row / DH, r = row % DH, wih = r / 32;
+  const int hs = row / DH, r = row % DH;
+  const int wig = half * (DH / 32) + r / 32;  // warp index inside the head group
   const int head = idx * HPT + hs;
-  if (head >= s.nq) return;  // whole warps: a ragged last tile has an empty head slot
+  const bool live = head < s.nq;  // whole warps: a ragged last tile has an empty head slot
+  float gq[HC];
+  if (live) {
+    const uint32_t tq = tacc + static_cast<uint32_t>(hs * DH + half * HC);
+#pragma unroll
+    for (int c0 = 0; c0 < HC; c0 += 32) {
+      uint32_t v[32];
+      tmem_ld32(tq + c0, v);
+#pragma unroll
+      for (int e = 0; e < 32; ++e) gq[c0 + e] = __uint_as_float(v[e]);
+    }
+    tmem_ld_wait();
+  }
+  tc_fence_before();
+  mbar_arrive(acce_bar);  // G_Q is in registers: the accumulator is free for the next tile
+  if (!live) return;
   const int bar = 1 + hs;
   const int g = head / s.G;
   const int tk = (g * DH) / 128, og = (g * DH) % 128;
   const unsigned* flag = a.flags + layer * s.tiles_k + tk;
-  if (r == 0) ep->ok[hs] = wait_flag(flag, a.epoch, abort, a.status) ? 1 : 0;
-  named_bar_sync(bar, DH);
+  if (r == 0 && half == 0) ep->ok[hs] = wait_flag(flag, a.epoch, abort, a.status) ? 1 : 0;
+  named_bar_sync(bar, NT);
   if (!ep->ok[hs]) return;
   (void)ld_acquire_u32(flag);
+  // Half row of G_K (stored transposed: element (j, r) is G_K[r][j]).
   const float* GK = a.gk + static_cast<size_t>(layer * s.tiles_k + tk) * 16384u + og * 128 + og;
-  float gk[DH];  // row r of G_K (stored transposed: element (j, r) is G_K[r][j])
+  float gk[HC];
 #pragma unroll
-  for (int j = 0; j < DH; ++j) gk[j] = __ldcg(GK + j * 128 + r);
+  for (int j = 0; j < HC; ++j) gk[j] = __ldcg(GK + (half * HC + j) * 128 + r);
   const size_t hidx = static_cast<size_t>(layer) * s.nq + head;
-  float z = __ldcg(a.z0 + (hidx * 2) * DH + r) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + r);
-  float* zs = ep->zs[hs];
-  float* ys = ep->ys[hs];
-  zs[r] = z;
-  named_bar_sync(bar, DH);
-  const uint32_t tq = tacc + static_cast<uint32_t>(hs * DH);
-  float sigma = 0.0f, inv_n = 0.0f, y = 0.0f;
+  float(*tsh)[128] = ep->tsh[hs];
+  float(*wsh)[128] = ep->wsh[hs];
+  wsh[half][r] = half == 0 ? __ldcg(a.z0 + (hidx * 2) * DH + r) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + r) : 0.0f;
+  named_bar_sync(bar, NT);
+  float c = 1.0f, sigma = 0.0f, y = 0.0f, n = 0.0f;
   for (int it = 0; it < a.iters; ++it) {
-    // t = G_Q z (row r);  sigma^2 = z . t;  y = t / sigma
+    // t' = G_Q x (this thread's half of row r);  S1 = x . t'
     float t0 = 0.0f, t1 = 0.0f, t2 = 0.0f, t3 = 0.0f;
 #pragma unroll
-    for (int c0 = 0; c0 < DH; c0 += 32) {
-      uint32_t v[32];
-      tmem_ld32(tq + c0, v);
-      tmem_ld_wait();
-#pragma unroll
-      for (int jj = 0; jj < 32; jj += 4) {
-        const float4 zz = *reinterpret_cast<const float4*>(zs + c0 + jj);
-        t0 = fmaf(__uint_as_float(v[jj + 0]), zz.x, t0);
-        t1 = fmaf(__uint_as_float(v[jj + 1]), zz.y, t1);
-        t2 = fmaf(__uint_as_float(v[jj + 2]), zz.z, t2);
-        t3 = fmaf(__uint_as_float(v[jj + 3]), zz.w, t3);
-      }
+    for (int j = 0; j < HC; j += 4) {
+      const float4 a0 = *reinterpret_cast<const float4*>(&wsh[0][half * HC + j]);
+      const float4 a1 = *reinterpret_cast<const float4*>(&wsh[1][half * HC + j]);
+      t0 = fmaf(gq[j + 0], a0.x + a1.x, t0);
+      t1 = fmaf(gq[j + 1], a0.y + a1.y, t1);
+      t2 = fmaf(gq[j + 2], a0.z + a1.z, t2);
+      t3 = fmaf(gq[j + 3], a0.w + a1.w, t3);
     }
-    const float t = (t0 + t1) + (t2 + t3);
-    float p = warp_sum(z * t);
-    if (lane == 0) ep->red[hs][0][wih] = p;
-    named_bar_sync(bar, DH);
-    float s2 = 0.0f;
+    const float tp = (t0 + t1) + (t2 + t3);
+    const float xr = wsh[0][r] + wsh[1][r];
+    tsh[half][r] = tp;
+    float p = warp_sum(xr * tp);
+    if (lane == 0) ep->red[hs][0][wig] = p;
+    named_bar_sync(bar, NT);
+    float s1 = 0.0f;
 #pragma unroll
-    for (int w = 0; w < WPH; ++w) s2 += ep->red[hs][0][w];
-    s2 = s2 < 0.0f ? 0.0f : s2;
-    sigma = sqrtf(s2);
-    const float inv_s = sigma > 0.0f ? 1.0f / sigma : 0.0f;
-    y = t * inv_s;
-    ys[r] = y;
-    named_bar_sync(bar, DH);
-    // w = G_K y (row r);  n^2 = y . w;  z = w / n
+    for (int w = 0; w < NW; ++w) s1 += ep->red[hs][0][w];
+    s1 = s1 < 0.0f ? 0.0f : s1;  // rounding can dip below 0; NaN must survive
+    const float rs1 = sqrtf(s1);
+    sigma = c > 0.0f ? rs1 / c : 0.0f;
+    const float inv1 = rs1 > 0.0f ? 1.0f / rs1 : 0.0f;
+    // w = G_K y with y = t' / sqrt(S1);  S2 = y . w
     float w0 = 0.0f, w1 = 0.0f, w2 = 0.0f, w3 = 0.0f;
 #pragma unroll
-    for (int j = 0; j < DH; j += 4) {
-      const float4 yy = *reinterpret_cast<const float4*>(ys + j);
-      w0 = fmaf(gk[j + 0], yy.x, w0);
-      w1 = fmaf(gk[j + 1], yy.y, w1);
-      w2 = fmaf(gk[j + 2], yy.z, w2);
-      w3 = fmaf(gk[j + 3], yy.w, w3);
+    for (int j = 0; j < HC; j += 4) {
+      const float4 b0 = *reinterpret_cast<const float4*>(&tsh[0][half * HC + j]);
+      const float4 b1 = *reinterpret_cast<const float4*>(&tsh[1][half * HC + j]);
+      w0 = fmaf(gk[j + 0], b0.x + b1.x, w0);
+      w1 = fmaf(gk[j + 1], b0.y + b1.y, w1);
+      w2 = fmaf(gk[j + 2], b0.z + b1.z, w2);
+      w3 = fmaf(gk[j + 3], b0.w + b1.w, w3);
     }
-    const float w = (w0 + w1) + (w2 + w3);
-    p = warp_sum(y * w);
-    if (lane == 0) ep->red[hs][1][wih] = p;
-    named_bar_sync(bar, DH);
-    float n2 = 0.0f;
+    const float wpart = ((w0 + w1) + (w2 + w3)) * inv1;
+    y = (tsh[0][r] + tsh[1][r]) * inv1;
+    wsh[half][r] = wpart;
+    p = warp_sum(y * wpart);
+    if (lane == 0) ep->red[hs][1][wig] = p;
+    named_bar_sync(bar, NT);
+    float s2 = 0.0f;
 #pragma unroll
-    for (int ww = 0; ww < WPH; ++ww) n2 += ep->red[hs][1][ww];
-    n2 = n2 < 0.0f ? 0.0f : n2;
-    const float n = sqrtf(n2);
-    inv_n = n > 0.0f ? 1.0f / n : 0.0f;
-    z = w * inv_n;
-    zs[r] = z;
-    named_bar_sync(bar, DH);
+    for (int w = 0; w < NW; ++w) s2 += ep->red[hs][1][w];
+    s2 = s2 < 0.0f ? 0.0f : s2;
+    n = sqrtf(s2);
+    c = n;
   }
-  a.ybuf[hidx * DH + r] = y * inv_n;
-  if (r == 0) {
+  if (half == 0) a.ybuf[hidx * DH + r] = n > 0.0f ? y / n : 0.0f;
+  if (r == 0 && half == 0) {
     a.sigma[hidx] = sigma;
     if (!isfinite(sigma)) set_status(a.status, GAS_DEV_NONFINITE_SIGMA);
     if (a.scale_out != nullptr) atomic_max_nonneg(&a.scale_out[layer], a.scale_c * sigma);
@@ -208,7 +232,8 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
 }
 
 template <int NZ, int DH, bool FUSED>
-__global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_constant__ GramArgs a) {
+__global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(const __grid_constant__ GramArgs a) {
+  constexpr int NE = 32 * GramWarps<FUSED>::kEpiWarps;  // epilogue threads
   using Cfg = GramCfg<NZ>;
   constexpr int S = Cfg::kStages;
   constexpr uint32_t SB = Cfg::kStageBytes;
@@ -235,7 +260,7 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
     }
     for (int i = 0; i < NA; ++i) {
       mbar_init(smem_u32(&accf[i]), 1);
-      mbar_init(smem_u32(&acce[i]), 128);
+      mbar_init(smem_u32(&acce[i]), NE);
     }
     mbar_init(smem_u32(done), 1);
     *abort = 0;
@@ -320,6 +345,8 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
     // ---------------- epilogue: TMEM -> global ----------------
     const int q = warp & 3;  // tcgen05.ld: warp w may read TMEM lanes 32*(w%4) .. +31
     const int row = q * 32 + lane;
+    const int half = (warp - 2) >> 2;  // fused: two threads per row, one per half of its columns
+    constexpr int CW = 128 * 128 / NE;  // accumulator columns per thread when storing G
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const int gpt = 128 / s.dh;
     uint32_t tc = 0;
@@ -328,28 +355,27 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
       const uint32_t acc = tc % NA, aph = (tc / NA) & 1u;
       const bool got = mbar_wait(smem_u32(&accf[acc]), aph, abort, a.status);
       __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the per-lane wait
-      // One decision for all four epilogue warps, so none of them can be left alone at
-      // a named barrier further down when another gave up.
-      if (!named_bar_and(4, 128, got)) break;
+      // One decision for all epilogue warps, so none of them can be left alone at a
+      // named barrier further down when another gave up.
+      if (!named_bar_and(4, NE, got)) break;
       tc_fence_after();
-      if (FUSED && !tr.is_k) {
-        fused_iterate<DH>(a, tr.layer, tr.idx, tmem + lane_off + acc * 128u, row, lane, ep, abort);
-        tc_fence_before();
-        mbar_arrive(smem_u32(&acce[acc]));
+      if (FUSED && !tr.is_k) {  // (hands the accumulator back itself, right after reading G_Q)
+        fused_iterate<DH>(a, tr.layer, tr.idx, tmem + lane_off + acc * 128u, row, half, lane, ep, abort,
+                          smem_u32(&acce[acc]));
         ++tc;
         continue;
       }
       float* Gout = (tr.is_k ? a.gk : a.gq) +
                     (static_cast<size_t>(tr.layer) * (tr.is_k ? s.tiles_k : s.tiles_q) + tr.idx) * 16384u;
 #pragma unroll 1
-      for (int c0 = 0; c0 < 128; c0 += 16) {
+      for (int c0 = half * CW; c0 < half * CW + CW; c0 += 16) {
         uint32_t r[16];
         tmem_ld16(tmem + lane_off + acc * 128u + c0, r);
         tmem_ld_wait();
 #pragma unroll
         for (int jj = 0; jj < 16; ++jj) Gout[(c0 + jj) * 128 + row] = __uint_as_float(r[jj]);
       }
-      if (tr.is_k) {
+      if (tr.is_k && half == 0) {
         const int gi = row / s.dh, i = row % s.dh;
         const int g = tr.idx * gpt + gi;
         const int twoG = 2 * s.G;
@@ -369,11 +395,11 @@ __global__ void __launch_bounds__(kGramThreads, 1) gram_kernel(const __grid_cons
             }
           }
         }
-        if (FUSED) {  // publish G_K and z0 of this key tile to the query tiles' epilogues
-          __threadfence();
-          named_bar_sync(3, 128);
-          if (row == 0) st_release_u32(a.flags + tr.layer * s.tiles_k + tr.idx, a.epoch);
-        }
+      }
+      if (FUSED && tr.is_k) {  // publish G_K and z0 of this key tile to the query tiles' epilogues
+        __threadfence();
+        named_bar_sync(3, NE);
+        if (row == 0 && half == 0) st_release_u32(a.flags + tr.layer * s.tiles_k + tr.idx, a.epoch);
       }
       tc_fence_before();
       mbar_arrive(smem_u32(&acce[acc]));
@@ -499,7 +525,7 @@ cudaError_t launch_gram_cfg(const GramArgs& a, int num_sms, cudaStream_t st) {
   const int grid = T < num_sms ? T : num_sms;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kGramThreads);
+  cfg.blockDim = dim3(GramWarps<FUSED>::kThreads);
   cfg.dynamicSmemBytes = Cfg::kSmem;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];

@@ -96,7 +96,7 @@ struct GramArgs {
   float scale_c;
 };
 
-// Tensor-core write-back v_out = B_g^T (y / ||v'||) for every head (group size <= 16).
+// Tensor-core write-back v_out = B_g^T (y / ||v'||) for every head.
 struct WbArgs {
   Shape s;
   const CUtensorMap* maps_k;  // [L] (box 64 x 128, as for the Gram pass)
@@ -135,6 +135,5 @@ cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st);
 cudaError_t launch_writeback(const WbArgs& a, int num_sms, cudaStream_t st);
 void set_global_error(const char* msg);  // message returned by gas_last_error(NULL)
 size_t gram_smem_bytes(int nz);
-constexpr int kWbMaxGroup = 16;  // tensor-core write-back handles n_q/n_kv <= 16
 
 }  // namespace gas

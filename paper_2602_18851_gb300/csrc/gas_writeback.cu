@@ -4,15 +4,15 @@
 //   v_out[h] = B_g^T (y_h / ||v'_h||)   for every head h of KV group g,
 //
 // one more pass over every key block B_g (d_h x d bf16).  Per key tile (128 rows = one
-// or two groups) and 64-column chunk c0.. of d it is one tcgen05 MMA chain
-//   D[n][c] = sum_i Y[n][i] * B[i][c],   M = 128 (n), N = 64 (c), K = 128 (i),
-// with A = Y split into bf16 hi and lo rows (about 16 bits of mantissa, K-major, staged
-// in shared memory by the epilogue warps) and B = the TMA box of the weight tile read
-// MN-major (its 64 contiguous columns are the N index).  Row layout of Y: head j of
-// group gi of the tile is number u = gi*G + j; it goes to TMEM lane quarter u % 4 (so
-// all four epilogue warps drain D), slot m = u / 4: hi part in row 32*(u%4) + m, lo part
-// in row 32*(u%4) + 16 + m, non-zero only in the group's own K range.  The epilogue adds
-// the hi and lo rows with one shuffle inside a warp.  Group size <= 16.
+// or two groups) and 128-column chunk c0.. of d it is one tcgen05 MMA chain
+//   D[c][n] = sum_i B[i][c] * Y[n][i],   M = 128 (c), N = nz (n), K = 128 (i),
+// with A = two TMA boxes of the weight tile read MN-major (their contiguous columns are
+// the M index) and B = Y, the vectors split into bf16 hi and lo rows (about 16 bits of
+// mantissa), K-major, staged in shared memory by the epilogue warps.  Row layout of Y:
+// head j of group gi of the tile is slot u = gi*G + j; its hi part is row u, its lo
+// part row nz/2 + u, non-zero only in the group's own K range.  Each epilogue thread
+// owns one column c (a TMEM lane) and adds rows u and nz/2 + u for every head, so a
+// warp writes 32 consecutive floats of each head's v_out row.
 
 #include "gas_device.cuh"
 
@@ -20,13 +20,25 @@ namespace gas {
 
 namespace {
 
-constexpr int kWbThreads = 192;            // warp 0 TMA, warp 1 MMA, warps 2-5 stage Y / drain D
-constexpr int kWbCols = 1024;              // columns of d per work item
-constexpr int kWbStages = 9;
-constexpr int kWbSlots = 4;                // tensor-memory accumulators of 64 columns
-constexpr uint32_t kBox = 128u * 64u * 2u; // 64 columns x 128 rows bf16
-constexpr uint32_t kYBytes = 2u * 16384u;  // 128 rows x 128 K bf16 as two 64-wide K atoms
-constexpr size_t kWbSmem = 2 * kYBytes + kWbStages * kBox + 4096;
+constexpr int kWbThreads = 192;               // warp 0 TMA, warp 1 MMA, warps 2-5 stage Y / drain D
+constexpr int kWbCols = 1024;                 // columns of d per work item
+constexpr int kWbSlots = 4;                   // tensor-memory accumulators of nz columns
+constexpr uint32_t kBox = 128u * 64u * 2u;    // 64 columns x 128 rows bf16
+constexpr uint32_t kStage = 2 * kBox;         // 128 columns
+constexpr int kWbSmemBudget = 232448;         // 227 KB opt-in dynamic shared memory
+
+template <int NZ>
+struct WbCfg {
+  static constexpr uint32_t kYBytes = 2u * NZ * 128u;  // nz rows x 128 K as two 64-wide K atoms
+  static constexpr int kStages =
+      (kWbSmemBudget - 4096 - 2 * static_cast<int>(kYBytes)) / static_cast<int>(kStage) > 6
+          ? 6
+          : (kWbSmemBudget - 4096 - 2 * static_cast<int>(kYBytes)) / static_cast<int>(kStage);
+  static constexpr size_t kSmem = 2 * kYBytes + kStages * kStage + 4096;
+  static constexpr uint32_t kTmemCols = (kWbSlots * NZ < 32) ? 32 : kWbSlots * NZ;
+  static_assert(kYBytes % 1024 == 0, "Y atoms must stay 1024-byte aligned");
+  static_assert(kStages >= 3, "ring too shallow");
+};
 
 struct WbItem {
   int layer, tile, c0, nchunks;
@@ -40,19 +52,21 @@ __device__ __forceinline__ WbItem decode_item(const Shape& s, int t) {
   w.tile = rem / ncb;
   w.c0 = (rem - w.tile * ncb) * kWbCols;
   const int ncols = min(kWbCols, s.d - w.c0);
-  w.nchunks = (ncols + 63) / 64;
+  w.nchunks = (ncols + 127) / 128;
   return w;
 }
 
-template <int DH>
+template <int DH, int NZ>
 __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_constant__ WbArgs a) {
-  constexpr int S = kWbStages;
+  using Cfg = WbCfg<NZ>;
+  constexpr int S = Cfg::kStages;
   constexpr int GPT = 128 / DH;  // groups per key tile
+  constexpr uint32_t YB = Cfg::kYBytes;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* ybuf_s = smem;                    // [2][kYBytes]
-  uint8_t* ring = smem + 2 * kYBytes;        // [S][kBox]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + S * kBox);
+  uint8_t* ring = smem;                      // [S][kStage]
+  uint8_t* ybuf_s = smem + S * kStage;       // [2][YB]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ybuf_s + 2 * YB);
   uint64_t* full = bars;
   uint64_t* empty = full + S;
   uint64_t* yfull = empty + S;
@@ -84,11 +98,11 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
     fence_mbar_init();
   }
   // Rows and K ranges of Y that no head uses stay zero for the whole launch.
-  for (uint32_t o = threadIdx.x * 16u; o < 2u * kYBytes; o += kWbThreads * 16u)
+  for (uint32_t o = threadIdx.x * 16u; o < 2u * YB; o += kWbThreads * 16u)
     *reinterpret_cast<uint4*>(ybuf_s + o) = make_uint4(0, 0, 0, 0);
   fence_proxy_async_smem();
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), 256);
+    tmem_alloc(smem_u32(tmem_slot), Cfg::kTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -109,8 +123,10 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           const uint32_t st = issued % S, ph = (issued / S) & 1u;
           if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1u, abort, a.status)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full[st]);
-          mbar_arrive_expect_tx(fb, kBox);
-          tma_load_2d(smem_u32(ring + st * kBox), &a.maps_k[w.layer], fb, w.c0 + 64 * j, w.tile * 128, pol);
+          const uint32_t dst = smem_u32(ring + st * kStage);
+          mbar_arrive_expect_tx(fb, kStage);
+          tma_load_2d(dst, &a.maps_k[w.layer], fb, w.c0 + 128 * j, w.tile * 128, pol);
+          tma_load_2d(dst + kBox, &a.maps_k[w.layer], fb, w.c0 + 128 * j + 64, w.tile * 128, pol);
           ++issued;
         }
       }
@@ -120,7 +136,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32_bmn(128, 64);
+      constexpr uint32_t idesc = idesc_bf16_f32_amn(128, NZ);
       uint32_t consumed = 0, cc = 0, it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x, ++it) {
@@ -128,19 +144,19 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
         const uint32_t yb = it & 1u;
         if (!mbar_wait(smem_u32(&yfull[yb]), (it >> 1) & 1u, abort, a.status)) break;
         tc_fence_after();
-        const uint32_t ybase = smem_u32(ybuf_s + yb * kYBytes);
+        const uint32_t ybase = smem_u32(ybuf_s + yb * YB);
         for (int j = 0; j < w.nchunks; ++j, ++cc) {
           const uint32_t slot = cc % kWbSlots;
           if (!mbar_wait(smem_u32(&dempty[slot]), ((cc / kWbSlots) & 1u) ^ 1u, abort, a.status)) { ok = false; break; }
           const uint32_t st = consumed % S, ph = (consumed / S) & 1u;
           if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t sx = smem_u32(ring + st * kBox);
+          const uint32_t sx = smem_u32(ring + st * kStage);
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            const uint64_t ad = desc_kmajor_sw128(ybase + (kk >> 2) * 16384u + (kk & 3) * 32u);
-            const uint64_t bd = desc_mnmajor_sw128(sx + kk * 2048u);
-            umma_bf16(tmem + slot * 64u, ad, bd, idesc, kk > 0 ? 1u : 0u);
+            const uint64_t ad = desc_mnmajor_sw128_2atoms(sx + kk * 2048u, kBox);
+            const uint64_t bd = desc_kmajor_sw128(ybase + (kk >> 2) * (YB / 2) + (kk & 3) * 32u);
+            umma_bf16(tmem + slot * NZ, ad, bd, idesc, kk > 0 ? 1u : 0u);
           }
           umma_commit(smem_u32(&empty[st]));
           umma_commit(smem_u32(&dfull[slot]));
@@ -156,7 +172,8 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
     const int ethr = threadIdx.x - 64;
     const int q = warp & 3;
     const int G = s.G;
-    const int units = GPT * G * (DH / 8);
+    const int nheads = GPT * G;  // head slots per key tile (<= NZ / 2)
+    const int units = nheads * (DH / 8);
     uint32_t staged = 0;
     // Stage Y (hi/lo bf16, swizzled K-major) of item t into buffer staged & 1.
     auto stage = [&](int t) -> bool {
@@ -164,16 +181,15 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
       const uint32_t yb = staged & 1u;
       const bool ok = mbar_wait(smem_u32(&yempty[yb]), ((staged >> 1) & 1u) ^ 1u, abort, a.status);
       if (ok) {
-        uint8_t* ybase = ybuf_s + yb * kYBytes;
-        for (int u = ethr; u < units; u += 128) {
-          const int gi = u / (G * (DH / 8));
-          const int rem = u - gi * G * (DH / 8);
-          const int j = rem / (DH / 8);
-          const int i0 = (rem - j * (DH / 8)) * 8;
+        uint8_t* ybase = ybuf_s + yb * YB;
+        for (int unit = ethr; unit < units; unit += 128) {
+          const int u = unit / (DH / 8);                  // head slot gi*G + j
+          const int i0 = (unit - u * (DH / 8)) * 8;
+          const int gi = u / G;
           const int g = w.tile * GPT + gi;
           float v[8];
           if (g < s.nkv) {
-            const float* src = a.ybuf + (static_cast<size_t>(w.layer) * s.nq + g * G + j) * DH + i0;
+            const float* src = a.ybuf + (static_cast<size_t>(w.layer) * s.nq + g * G + (u - gi * G)) * DH + i0;
             const float4 a0 = *reinterpret_cast<const float4*>(src);
             const float4 a1 = *reinterpret_cast<const float4*>(src + 4);
             v[0] = a0.x; v[1] = a0.y; v[2] = a0.z; v[3] = a0.w;
@@ -188,11 +204,10 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
             hb[e] = f32_to_bf16_bits(v[e]);
             lb[e] = f32_to_bf16_bits(v[e] - __uint_as_float(hb[e] << 16));
           }
-          const int k = gi * DH + i0;                 // K index of the 8-element chunk
+          const int k = gi * DH + i0;                     // K index of the 8-element chunk
           const int region = k >> 6, chunk = (k & 63) >> 3;
-          const int hu = gi * G + j;                  // head slot u -> quarter u%4, row u/4
-          const int rhi = 32 * (hu & 3) + (hu >> 2), rlo = rhi + 16;
-          uint8_t* base = ybase + region * 16384;
+          const int rhi = u, rlo = NZ / 2 + u;
+          uint8_t* base = ybase + region * (YB / 2);
           *reinterpret_cast<uint4*>(base + rhi * 128 + ((chunk ^ (rhi & 7)) << 4)) =
               make_uint4(hb[0] | (hb[1] << 16), hb[2] | (hb[3] << 16), hb[4] | (hb[5] << 16), hb[6] | (hb[7] << 16));
           *reinterpret_cast<uint4*>(base + rlo * 128 + ((chunk ^ (rlo & 7)) << 4)) =
@@ -218,27 +233,27 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
         __syncwarp();
         if (!named_bar_and(4, 128, got)) { ok = false; break; }
         tc_fence_after();
-        if (q < GPT * G) {  // this lane quarter holds at least one head
-          uint32_t r0[32], r1[32];
-          const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + slot * 64u;
-          tmem_ld32(taddr, r0);
-          tmem_ld32(taddr + 32u, r1);
+        const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + slot * NZ;
+        const int col = w.c0 + 128 * j + q * 32 + lane;
+#pragma unroll
+        for (int n0 = 0; n0 < NZ / 2; n0 += 16) {  // hi rows n0.., lo rows NZ/2 + n0..
+          uint32_t hi[16], lo[16];
+          tmem_ld16(taddr + n0, hi);
+          tmem_ld16(taddr + NZ / 2 + n0, lo);
           tmem_ld_wait();
-          float o[64];
+          if (col < s.d) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            const float hi0 = __uint_as_float(r0[c]), hi1 = __uint_as_float(r1[c]);
-            o[c] = hi0 + __shfl_down_sync(0xFFFFFFFFu, hi0, 16);
-            o[32 + c] = hi1 + __shfl_down_sync(0xFFFFFFFFu, hi1, 16);
-          }
-          const int hu = 4 * lane + q;  // head slot held by this lane's hi row
-          const int g = w.tile * GPT + hu / G;
-          if (lane < 16 && hu < GPT * G && g < s.nkv) {
-            const int col0 = w.c0 + 64 * j;
-            float* dst = a.v_out + (static_cast<size_t>(w.layer) * s.nq + g * G + hu % G) * s.d + col0;
-#pragma unroll
-            for (int c = 0; c < 64; c += 4)
-              if (col0 + c < s.d) *reinterpret_cast<float4*>(dst + c) = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+            for (int e = 0; e < 16; ++e) {
+              const int u = n0 + e;
+              if (u < nheads) {
+                const int gi = u / G;
+                const int g = w.tile * GPT + gi;
+                if (g < s.nkv) {
+                  const size_t h = static_cast<size_t>(w.layer) * s.nq + g * G + (u - gi * G);
+                  a.v_out[h * s.d + col] = __uint_as_float(hi[e]) + __uint_as_float(lo[e]);
+                }
+              }
+            }
           }
         }
         tc_fence_before();
@@ -251,30 +266,41 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem, 256);
+    tmem_dealloc(tmem, Cfg::kTmemCols);
   }
 }
 
-template <int DH>
-cudaError_t launch_wb_dh(const WbArgs& a, int num_sms, cudaStream_t st) {
+template <int DH, int NZ>
+cudaError_t launch_wb_cfg(const WbArgs& a, int num_sms, cudaStream_t st) {
+  using Cfg = WbCfg<NZ>;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(writeback_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(kWbSmem));
+    cudaError_t e = cudaFuncSetAttribute(writeback_kernel<DH, NZ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(Cfg::kSmem));
     if (e != cudaSuccess) return e;
     configured = true;
   }
   const int ncb = (a.s.d + kWbCols - 1) / kWbCols;
   const int T = a.s.L * a.s.tiles_k * ncb;
   const int grid = T < num_sms ? T : num_sms;
-  writeback_kernel<DH><<<grid, kWbThreads, kWbSmem, st>>>(a);
+  writeback_kernel<DH, NZ><<<grid, kWbThreads, Cfg::kSmem, st>>>(a);
   return cudaGetLastError();
+}
+
+template <int DH>
+cudaError_t launch_wb_dh(const WbArgs& a, int num_sms, cudaStream_t st) {
+  switch (a.s.nz) {
+    case 16: return launch_wb_cfg<DH, 16>(a, num_sms, st);
+    case 32: return launch_wb_cfg<DH, 32>(a, num_sms, st);
+    case 64: return launch_wb_cfg<DH, 64>(a, num_sms, st);
+    case 128: return launch_wb_cfg<DH, 128>(a, num_sms, st);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace
 
 cudaError_t launch_writeback(const WbArgs& a, int num_sms, cudaStream_t st) {
-  if (a.s.G > kWbMaxGroup) return cudaErrorInvalidValue;
   if (a.s.dh == 128) return launch_wb_dh<128>(a, num_sms, st);
   if (a.s.dh == 64) return launch_wb_dh<64>(a, num_sms, st);
   return cudaErrorInvalidValue;

@@ -71,8 +71,8 @@ WORKLOADS = {
     "tiny-gqa128": Workload("tiny-gqa128", 3, 512, 8, 2, 128, 15, "spike4", _BASE_SEED + 13),
     "ragged": Workload("ragged", 3, 200, 6, 3, 64, 10, "lognormal", _BASE_SEED + 14),
     "ragged128": Workload("ragged128", 2, 1000, 5, 5, 128, 9, "spike1", _BASE_SEED + 15),
-    # Group-size edge cases: 16 query heads per KV head (largest tensor-core write-back
-    # group) and 32 (write-back falls back to CUDA cores; widest z0 operand).
+    # Group-size edge cases: 16 and 32 query heads per KV head (the latter gives the
+    # widest z0 / write-back operand, 128 rows).
     "tiny-g16": Workload("tiny-g16", 2, 384, 16, 1, 128, 8, "spike4", _BASE_SEED + 16),
     "tiny-g32": Workload("tiny-g32", 2, 320, 32, 1, 64, 8, "spike4", _BASE_SEED + 17),
 }
