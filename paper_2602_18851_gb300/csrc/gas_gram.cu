@@ -32,7 +32,7 @@ struct GramWarps {
 };
 constexpr uint32_t kTileBytes = 128u * 64u * 2u;  // one 128-row x 64-column bf16 box
 constexpr int kSmemBudget = 232448;               // 227 KB opt-in dynamic shared memory
-constexpr int kSmemReserve = 6144;                // alignment slack, barriers, epilogue scratch
+constexpr int kSmemReserve = 22528;               // alignment slack, barriers, epilogue scratch
 
 template <int NZ>
 struct GramCfg {
@@ -109,122 +109,187 @@ __device__ __forceinline__ TileRef decode_tile(const Shape& s, int t) {
   return r;
 }
 
-// Shared scratch of the fused epilogue, per head slot of a tile (two heads per tile
-// when d_h = 64): the half-row partial sums of t' = G_Q x and of w = G_K y written by
-// the two thread halves, and the per-warp partial dot products.
+// Shared scratch of the fused epilogue.  `stage` carries one TMEM lane quarter (32 rows)
+// of a query tile's G_Q at a time from the row-per-thread layout tcgen05.ld produces to
+// the block layout of the iteration; xs / ts hold the current x and t' of each head
+// slot (two heads per tile when d_h = 64); red the per-warp partial dot products.
 struct EpiSmem {
-  float tsh[2][2][128];  // [slot][half][row]
-  float wsh[2][2][128];
-  float red[2][2][8];    // [slot][which dot][warp of the head group]
+  float stage[32][129];
+  float xs[2][128];
+  float ts[2][128];
+  float red[2][2][8];  // [slot][which dot][warp of the head group]
   int ok[2];
 };
 
-// k power iterations for the head(s) of one query tile in R^{d_h}.  Each row r of the
-// head's d_h x d_h block is held by two threads (half = 0, 1), each with half of the
-// row of G_Q (read once from the tile's tensor-memory accumulator, which is then handed
-// back to the MMA warp) and half of the row of G_K (published by the key tile).
+// Sum over the 16 lanes of a half-warp of 8 values per lane: on return v[0] holds the
+// total of value number `idx` (3 halving exchange steps plus one butterfly step).
+__device__ __forceinline__ float halfwarp_transpose_reduce8(float (&v)[8], int lane, int& idx) {
+  int base = 0;
+#pragma unroll
+  for (int n = 8, off = 8; n > 1; n >>= 1, off >>= 1) {
+    const int h = n >> 1;
+    const bool up = (lane & off) != 0;
+#pragma unroll
+    for (int k = 0; k < h; ++k) {
+      const float send = up ? v[k] : v[k + h];
+      const float keep = up ? v[k + h] : v[k];
+      v[k] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, off);
+    }
+    if (up) base += h;
+  }
+  v[0] += __shfl_xor_sync(0xFFFFFFFFu, v[0], 1);
+  idx = base;
+  return v[0];
+}
+
+// k power iterations for the head(s) of one query tile, in R^{d_h}, run by the 8
+// epilogue warps.  Block layout: inside a head, warp w owns rows 16w + 8*(lane/16) .. +8
+// and lane % 16 owns d_h/16 consecutive columns, for both G_Q (copied once out of the
+// tile's tensor-memory accumulator, which is then handed back to the MMA warp) and G_K
+// (published by the key tile).  A matvec is 8 x d_h/16 FMAs per thread plus an 8-value
+// half-warp reduction; each thread reads only its own d_h/16 entries of the vector.
 // With x = c z (c a known scalar, c = 1 for z0) one iteration of Algorithm 2 is
 //   t' = G_Q x,  S1 = x.t' = c^2 sigma^2,  y = t' / sqrt(S1),
 //   w  = G_K y,  S2 = y.w = ||v'||^2,       x <- w,  c <- sqrt(S2),
-// so only two barriers per iteration are needed (after t' and after w).
+// two barriers per iteration.
 template <int DH>
-__device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int idx, uint32_t tacc, int row,
-                                              int half, int lane, EpiSmem* ep, volatile int* abort,
+__device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int idx, uint32_t tacc, int q,
+                                              int half, int ew, int lane, EpiSmem* ep, volatile int* abort,
                                               uint32_t acce_bar) {
   constexpr int HPT = 128 / DH;   // heads per 128-row tile
-  constexpr int HC = DH / 2;      // columns per thread (half a row)
-  constexpr int NT = 2 * DH;      // threads per head
-  constexpr int NW = NT / 32;     // warps per head
+  constexpr int NTH = 256 / HPT;  // threads per head
+  constexpr int NWH = NTH / 32;   // warps per head
+  constexpr int CPT = DH / 16;    // columns per thread
+  constexpr int HALF = DH / 2;    // accumulator columns each loader thread copies
   const Shape& s = a.s;
-  const int hs = row / DH, r = row % DH;
-  const int wig = half * (DH / 32) + r / 32;  // warp index inside the head group
-  const int head = idx * HPT + hs;
-  const bool live = head < s.nq;  // whole warps: a ragged last tile has an empty head slot
-  float gq[HC];
-  if (live) {
-    const uint32_t tq = tacc + static_cast<uint32_t>(hs * DH + half * HC);
+  // (1) copy this thread's TMEM row (its head block, its half of the columns) to registers
+  const int trow = q * 32 + lane;                 // tile row = TMEM lane
+  const int lslot = trow / DH;                    // head slot of that row
+  float rowv[HALF];
+  {
+    const uint32_t ta = tacc + static_cast<uint32_t>(lslot * DH + half * HALF);
 #pragma unroll
-    for (int c0 = 0; c0 < HC; c0 += 32) {
+    for (int c0 = 0; c0 < HALF; c0 += 32) {
       uint32_t v[32];
-      tmem_ld32(tq + c0, v);
+      tmem_ld32(ta + c0, v);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) gq[c0 + e] = __uint_as_float(v[e]);
+      for (int e = 0; e < 32; ++e) rowv[c0 + e] = __uint_as_float(v[e]);
     }
     tmem_ld_wait();
   }
   tc_fence_before();
   mbar_arrive(acce_bar);  // G_Q is in registers: the accumulator is free for the next tile
-  if (!live) return;
+  // (2) re-distribute G_Q into the block layout, one lane quarter at a time
+  const int hs = ew / NWH, ewh = ew % NWH;
+  const int rs = lane >> 4, cg = lane & 15;
+  const int rb = 16 * ewh + 8 * rs;               // first of my 8 rows inside the head block
+  const int cb = CPT * cg;                        // first of my columns
+  const int myq = (hs * DH + rb) >> 5;            // lane quarter holding my rows
+  float gq[8][CPT];
+#pragma unroll 1
+  for (int qq = 0; qq < 4; ++qq) {
+    if (q == qq) {
+#pragma unroll
+      for (int c = 0; c < HALF; ++c) ep->stage[lane][half * HALF + c] = rowv[c];
+    }
+    named_bar_sync(5, 256);
+    if (myq == qq) {
+      const int r0 = hs * DH + rb - 32 * qq;
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int k = 0; k < CPT; ++k) gq[i][k] = ep->stage[r0 + i][cb + k];
+    }
+    named_bar_sync(5, 256);
+  }
+  const int head = idx * HPT + hs;
+  if (head >= s.nq) return;  // whole head groups: a ragged last tile has an empty slot
+  // (3) wait for the key tile, then G_K (block layout) and z0
   const int bar = 1 + hs;
+  const int th = ewh * 32 + lane;                 // thread index inside the head group
   const int g = head / s.G;
   const int tk = (g * DH) / 128, og = (g * DH) % 128;
   const unsigned* flag = a.flags + layer * s.tiles_k + tk;
-  if (r == 0 && half == 0) ep->ok[hs] = wait_flag(flag, a.epoch, abort, a.status) ? 1 : 0;
-  named_bar_sync(bar, NT);
+  if (th == 0) ep->ok[hs] = wait_flag(flag, a.epoch, abort, a.status) ? 1 : 0;
+  named_bar_sync(bar, NTH);
   if (!ep->ok[hs]) return;
   (void)ld_acquire_u32(flag);
-  // Half row of G_K (stored transposed: element (j, r) is G_K[r][j]).
+  // G_K is stored transposed: element (j, i) holds G_K[i][j]; rows rb.. are contiguous.
   const float* GK = a.gk + static_cast<size_t>(layer * s.tiles_k + tk) * 16384u + og * 128 + og;
-  float gk[HC];
+  float gk[8][CPT];
 #pragma unroll
-  for (int j = 0; j < HC; ++j) gk[j] = __ldcg(GK + (half * HC + j) * 128 + r);
+  for (int k = 0; k < CPT; ++k) {
+    const float4 a0 = __ldcg(reinterpret_cast<const float4*>(GK + (cb + k) * 128 + rb));
+    const float4 a1 = __ldcg(reinterpret_cast<const float4*>(GK + (cb + k) * 128 + rb + 4));
+    gk[0][k] = a0.x; gk[1][k] = a0.y; gk[2][k] = a0.z; gk[3][k] = a0.w;
+    gk[4][k] = a1.x; gk[5][k] = a1.y; gk[6][k] = a1.z; gk[7][k] = a1.w;
+  }
   const size_t hidx = static_cast<size_t>(layer) * s.nq + head;
-  float(*tsh)[128] = ep->tsh[hs];
-  float(*wsh)[128] = ep->wsh[hs];
-  wsh[half][r] = half == 0 ? __ldcg(a.z0 + (hidx * 2) * DH + r) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + r) : 0.0f;
-  named_bar_sync(bar, NT);
+  float* xs = ep->xs[hs];
+  float* ts = ep->ts[hs];
+  if (th < DH) xs[th] = __ldcg(a.z0 + (hidx * 2) * DH + th) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + th);
+  named_bar_sync(bar, NTH);
+  const bool writer = (lane & 1) == 0;            // one of the two lanes holding a row total
   float c = 1.0f, sigma = 0.0f, y = 0.0f, n = 0.0f;
+  int ridx = 0;
   for (int it = 0; it < a.iters; ++it) {
-    // t' = G_Q x (this thread's half of row r);  S1 = x . t'
-    float t0 = 0.0f, t1 = 0.0f, t2 = 0.0f, t3 = 0.0f;
+    // t' = G_Q x;  S1 = x . t'
+    float xv[CPT];
 #pragma unroll
-    for (int j = 0; j < HC; j += 4) {
-      const float4 a0 = *reinterpret_cast<const float4*>(&wsh[0][half * HC + j]);
-      const float4 a1 = *reinterpret_cast<const float4*>(&wsh[1][half * HC + j]);
-      t0 = fmaf(gq[j + 0], a0.x + a1.x, t0);
-      t1 = fmaf(gq[j + 1], a0.y + a1.y, t1);
-      t2 = fmaf(gq[j + 2], a0.z + a1.z, t2);
-      t3 = fmaf(gq[j + 3], a0.w + a1.w, t3);
+    for (int k = 0; k < CPT; k += 4) {
+      const float4 x4 = *reinterpret_cast<const float4*>(xs + cb + k);
+      xv[k] = x4.x; xv[k + 1] = x4.y; xv[k + 2] = x4.z; xv[k + 3] = x4.w;
     }
-    const float tp = (t0 + t1) + (t2 + t3);
-    const float xr = wsh[0][r] + wsh[1][r];
-    tsh[half][r] = tp;
-    float p = warp_sum(xr * tp);
-    if (lane == 0) ep->red[hs][0][wig] = p;
-    named_bar_sync(bar, NT);
+    float part[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      float acc0 = 0.0f;
+#pragma unroll
+      for (int k = 0; k < CPT; ++k) acc0 = fmaf(gq[i][k], xv[k], acc0);
+      part[i] = acc0;
+    }
+    const float tp = halfwarp_transpose_reduce8(part, lane, ridx);
+    const int row = rb + ridx;
+    const float xr = xs[row];
+    if (writer) ts[row] = tp;
+    float p = warp_sum(writer ? xr * tp : 0.0f);
+    if (lane == 0) ep->red[hs][0][ewh] = p;
+    named_bar_sync(bar, NTH);
     float s1 = 0.0f;
 #pragma unroll
-    for (int w = 0; w < NW; ++w) s1 += ep->red[hs][0][w];
+    for (int w = 0; w < NWH; ++w) s1 += ep->red[hs][0][w];
     s1 = s1 < 0.0f ? 0.0f : s1;  // rounding can dip below 0; NaN must survive
     const float rs1 = sqrtf(s1);
     sigma = c > 0.0f ? rs1 / c : 0.0f;
     const float inv1 = rs1 > 0.0f ? 1.0f / rs1 : 0.0f;
-    // w = G_K y with y = t' / sqrt(S1);  S2 = y . w
-    float w0 = 0.0f, w1 = 0.0f, w2 = 0.0f, w3 = 0.0f;
+    // w = G_K y with y = t' / sqrt(S1);  S2 = y . w;  next x = w
 #pragma unroll
-    for (int j = 0; j < HC; j += 4) {
-      const float4 b0 = *reinterpret_cast<const float4*>(&tsh[0][half * HC + j]);
-      const float4 b1 = *reinterpret_cast<const float4*>(&tsh[1][half * HC + j]);
-      w0 = fmaf(gk[j + 0], b0.x + b1.x, w0);
-      w1 = fmaf(gk[j + 1], b0.y + b1.y, w1);
-      w2 = fmaf(gk[j + 2], b0.z + b1.z, w2);
-      w3 = fmaf(gk[j + 3], b0.w + b1.w, w3);
+    for (int k = 0; k < CPT; k += 4) {
+      const float4 t4 = *reinterpret_cast<const float4*>(ts + cb + k);
+      xv[k] = t4.x; xv[k + 1] = t4.y; xv[k + 2] = t4.z; xv[k + 3] = t4.w;
     }
-    const float wpart = ((w0 + w1) + (w2 + w3)) * inv1;
-    y = (tsh[0][r] + tsh[1][r]) * inv1;
-    wsh[half][r] = wpart;
-    p = warp_sum(y * wpart);
-    if (lane == 0) ep->red[hs][1][wig] = p;
-    named_bar_sync(bar, NT);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      float acc0 = 0.0f;
+#pragma unroll
+      for (int k = 0; k < CPT; ++k) acc0 = fmaf(gk[i][k], xv[k], acc0);
+      part[i] = acc0;
+    }
+    const float wrow = halfwarp_transpose_reduce8(part, lane, ridx) * inv1;
+    y = tp * inv1;
+    if (writer) xs[row] = wrow;
+    p = warp_sum(writer ? y * wrow : 0.0f);
+    if (lane == 0) ep->red[hs][1][ewh] = p;
+    named_bar_sync(bar, NTH);
     float s2 = 0.0f;
 #pragma unroll
-    for (int w = 0; w < NW; ++w) s2 += ep->red[hs][1][w];
+    for (int w = 0; w < NWH; ++w) s2 += ep->red[hs][1][w];
     s2 = s2 < 0.0f ? 0.0f : s2;
     n = sqrtf(s2);
     c = n;
   }
-  if (half == 0) a.ybuf[hidx * DH + r] = n > 0.0f ? y / n : 0.0f;
-  if (r == 0 && half == 0) {
+  if (writer && a.iters > 0) a.ybuf[hidx * DH + rb + ridx] = n > 0.0f ? y / n : 0.0f;
+  if (th == 0) {
     a.sigma[hidx] = sigma;
     if (!isfinite(sigma)) set_status(a.status, GAS_DEV_NONFINITE_SIGMA);
     if (a.scale_out != nullptr) atomic_max_nonneg(&a.scale_out[layer], a.scale_c * sigma);
@@ -360,8 +425,8 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       if (!named_bar_and(4, NE, got)) break;
       tc_fence_after();
       if (FUSED && !tr.is_k) {  // (hands the accumulator back itself, right after reading G_Q)
-        fused_iterate<DH>(a, tr.layer, tr.idx, tmem + lane_off + acc * 128u, row, half, lane, ep, abort,
-                          smem_u32(&acce[acc]));
+        fused_iterate<DH>(a, tr.layer, tr.idx, tmem + lane_off + acc * 128u, q, half, warp - 2, lane, ep,
+                          abort, smem_u32(&acce[acc]));
         ++tc;
         continue;
       }
