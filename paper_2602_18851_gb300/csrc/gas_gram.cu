@@ -99,13 +99,20 @@ struct TileRef {
   int layer, is_k, idx;
 };
 
+// Tile order: every key tile of every layer first, then the query tiles layer by layer,
+// so that a query tile's epilogue finds its key tile's G_K and z0 long published.
 __device__ __forceinline__ TileRef decode_tile(const Shape& s, int t) {
-  const int tpl = s.tiles_k + s.tiles_q;
   TileRef r;
-  r.layer = t / tpl;
-  const int rem = t - r.layer * tpl;
-  r.is_k = rem < s.tiles_k;
-  r.idx = r.is_k ? rem : rem - s.tiles_k;
+  const int nk = s.L * s.tiles_k;
+  r.is_k = t < nk;
+  if (r.is_k) {
+    r.layer = t / s.tiles_k;
+    r.idx = t - r.layer * s.tiles_k;
+  } else {
+    const int u = t - nk;
+    r.layer = u / s.tiles_q;
+    r.idx = u - r.layer * s.tiles_q;
+  }
   return r;
 }
 
@@ -260,8 +267,9 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
     for (int w = 0; w < NWH; ++w) s1 += ep->red[hs][0][w];
     s1 = s1 < 0.0f ? 0.0f : s1;  // rounding can dip below 0; NaN must survive
     const float rs1 = sqrtf(s1);
-    sigma = c > 0.0f ? rs1 / c : 0.0f;
-    const float inv1 = rs1 > 0.0f ? 1.0f / rs1 : 0.0f;
+    // zero guards that let a NaN through (x == 0 tests are false for NaN)
+    sigma = c == 0.0f ? 0.0f : rs1 / c;
+    const float inv1 = rs1 == 0.0f ? 0.0f : 1.0f / rs1;
     // w = G_K y with y = t' / sqrt(S1);  S2 = y . w;  next x = w
 #pragma unroll
     for (int k = 0; k < CPT; k += 4) {
@@ -288,7 +296,7 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
     n = sqrtf(s2);
     c = n;
   }
-  if (writer && a.iters > 0) a.ybuf[hidx * DH + rb + ridx] = n > 0.0f ? y / n : 0.0f;
+  if (writer && a.iters > 0) a.ybuf[hidx * DH + rb + ridx] = n == 0.0f ? 0.0f : y / n;
   if (th == 0) {
     a.sigma[hidx] = sigma;
     if (!isfinite(sigma)) set_status(a.status, GAS_DEV_NONFINITE_SIGMA);
@@ -537,7 +545,7 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
     s2 = warp_sum(s2);
     s2 = s2 < 0.0f ? 0.0f : s2;  // rounding can dip below 0; NaN must survive
     sigma = sqrtf(s2);
-    const float inv_s = sigma > 0.0f ? 1.0f / sigma : 0.0f;
+    const float inv_s = sigma == 0.0f ? 0.0f : 1.0f / sigma;
 #pragma unroll
     for (int c = 0; c < CPL; ++c) y[c] = t[c] * inv_s;
     // w = G_K y  (= B v');  n^2 = y . w (= ||v'||^2);  z = w / n (= B v)
@@ -560,7 +568,7 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
     n2 = warp_sum(n2);
     n2 = n2 < 0.0f ? 0.0f : n2;
     const float n = sqrtf(n2);
-    inv_n = n > 0.0f ? 1.0f / n : 0.0f;
+    inv_n = n == 0.0f ? 0.0f : 1.0f / n;
 #pragma unroll
     for (int c = 0; c < CPL; ++c) z[c] = wv[c] * inv_n;
   }
