@@ -129,6 +129,23 @@ gas_status gas_refresh(gas_handle h, const void *const *wq, const void *const *w
                        const float *v_in, float *v_out, float *sigma, double gamma,
                        double delta_star, double r_max, float *s, void *stream);
 
+/*
+ * Whole-layer spectral norm, Algorithms 2-3 (Appendix E) as printed: one persistent v
+ * per layer and M = W^Q W^K_exp^T with W^Q = all n_q heads ([d x n_q*d_h]) and W^K_exp
+ * the RepeatBlocks expansion of W^K (Section 4.2, never formed: RepeatBlocks / SumGroups
+ * act on the n_kv*d_h-vectors).  sigma_l = ||u'|| of the last iteration.
+ *   v_in, v_out : device fp32 [layers][d] (v_out may alias v_in or be NULL).
+ *   sigma       : device fp32 [layers].
+ *   s           : device fp32 [layers] or NULL; if given, the layer scale of Eq. 15 with
+ *                 sigma_l (gamma, delta_star, r_max as for gas_scales).
+ * Each iteration streams W^Q and W^K twice (no d_h x d_h reduction exists for the
+ * n_q*d_h-dimensional inner space).  Errors as gas_refresh; GAS_ERR_UNSUPPORTED when
+ * d or n_q*d_h exceeds what one CTA's shared memory holds (about 57000 floats).
+ */
+gas_status gas_layer_refresh(gas_handle h, const void *const *wq, const void *const *wk, int iters,
+                             const float *v_in, float *v_out, float *sigma, double gamma,
+                             double delta_star, double r_max, float *s, void *stream);
+
 /* Host helpers in float64: Eq. 12 (smallest gamma > 1; 1.0 if the bound holds for
  * every gamma; NaN on invalid input) and Eq. 13 (alpha_min for a given gamma). */
 double gas_gamma_min(int d_h, long long n_heads_total, int seq_len, double delta_star);

@@ -99,6 +99,7 @@ def load(path: str = LIB_PATH):
     lib.gas_last_launch_name.argtypes = [vp, c_int]
     lib.gas_last_launch_name.restype = ctypes.c_char_p
     lib.gas_spectral_norms_static.argtypes = [c_int] * 5 + [vp, vp, c_int, vp, vp, vp, vp]
+    lib.gas_layer_refresh.argtypes = [vp, vp, vp, c_int, vp, vp, vp, c_double, c_double, c_double, vp, vp]
     _lib = lib
     return lib
 
@@ -265,6 +266,31 @@ class Handle:
                                 v_out.data_ptr() if v_out is not None else None, sigma.data_ptr(),
                                 float(gamma), float(delta_star), float(r_max), s.data_ptr(),
                                 _stream_ptr(stream))
+        _check(st, self._h)
+        return sigma, s, v_out
+
+
+    def layer_refresh(self, wq, wk, iters: int, v_in: torch.Tensor, v_out: Optional[torch.Tensor] = None,
+                      sigma: Optional[torch.Tensor] = None, s: Optional[torch.Tensor] = None,
+                      gamma: float = 0.0, delta_star: float = 1e-6, r_max: float = E4M3_MAX,
+                      write_back: bool = True, with_scales: bool = True, stream=None):
+        """Whole-layer sigma_l = ||W^Q W^K_exp^T||_2 (Algorithms 2-3 over all heads), one v
+        per layer: v_in [layers, d].  Returns (sigma[layers], s[layers] or None, v_out)."""
+        qa = _ptr_array(wq, self.n_q * self.d_h, self.d, "wq")
+        ka = _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk")
+        shape = (self.layers, self.d)
+        if v_in.dtype != torch.float32 or tuple(v_in.shape) != shape or not v_in.is_contiguous():
+            raise ValueError(f"v_in must be a contiguous float32 tensor of shape {shape}")
+        if v_out is None and write_back:
+            v_out = torch.empty_like(v_in)
+        if sigma is None:
+            sigma = torch.empty(self.layers, device=v_in.device, dtype=torch.float32)
+        if s is None and with_scales:
+            s = torch.empty(self.layers, device=v_in.device, dtype=torch.float32)
+        st = load().gas_layer_refresh(self._h, qa, ka, int(iters), v_in.data_ptr(),
+                                      v_out.data_ptr() if v_out is not None else None, sigma.data_ptr(),
+                                      float(gamma), float(delta_star), float(r_max),
+                                      s.data_ptr() if s is not None else None, _stream_ptr(stream))
         _check(st, self._h)
         return sigma, s, v_out
 

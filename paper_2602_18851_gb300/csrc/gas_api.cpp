@@ -47,6 +47,10 @@ struct gas_ctx {
   float* ybuf = nullptr;
   CUtensorMap* dmaps = nullptr;  // [2L + 1]: q maps, k maps, v map
   unsigned* flags = nullptr;     // [L][tiles_k] key-tile flags of the fused kernel
+  float* lz = nullptr;           // whole-layer path: z_kv [L][n_kv*d_h]
+  float* lu = nullptr;           //                   u'   [L][d]
+  float* ly = nullptr;           //                   y    [L][n_q*d_h]
+  float* lv = nullptr;           //                   v'   [L][d]
   unsigned epoch = 0;            // last flag value used
 
   // host copies of the encoded descriptors and the pointers they were built for
@@ -323,6 +327,65 @@ gas_status spectral_impl(gas_ctx* h, const void* const* wq, const void* const* w
   return run_gram(h, wq, wk, tab, iters, v_in, v_out, sigma, s_out, scale_c, method == GAS_METHOD_FUSED, st);
 }
 
+// Whole-layer sigma (Algorithms 2-3 over all heads of a layer): 4 streaming kernels per
+// iteration, then sigma = ||u'||, v_out = v'/||v'|| and the layer scale.
+gas_status run_layer(gas_ctx* h, const gas::LayerTable& tab, int iters, const float* v_in, float* v_out,
+                     float* sigma, float* s_out, float scale_c, cudaStream_t st) {
+  const Shape& s = h->s;
+  const size_t Rq = static_cast<size_t>(s.nq) * s.dh, Rk = static_cast<size_t>(s.nkv) * s.dh;
+  int launches = 0;
+  cudaError_t e = cudaSuccess;
+  for (int it = 0; it < iters && e == cudaSuccess; ++it) {
+    gas::LayerArgs a{};
+    a.s = s;
+    a.which = 0;  // z_kv = W^K^T (v/||v||)
+    a.src = it == 0 ? v_in : h->lv;
+    a.out = h->lz;
+    a.out_stride = Rk;
+    e = launch(h, "layer_rowdot_k", st, [&] { return gas::launch_layer_rowdot(tab, a, st); });
+    ++launches;
+    if (e != cudaSuccess) break;
+    a.which = 1;  // u' = W^Q RepeatBlocks(z_kv)
+    a.src = h->lz;
+    a.src_stride = Rk;
+    a.out = h->lu;
+    a.out_stride = s.d;
+    e = launch(h, "layer_coldot_q", st, [&] { return gas::launch_layer_coldot(tab, a, st); });
+    ++launches;
+    if (e != cudaSuccess || (it == iters - 1 && v_out == nullptr)) break;
+    a.which = 1;  // y = W^Q^T (u'/||u'||)
+    a.src = h->lu;
+    a.out = h->ly;
+    a.out_stride = Rq;
+    e = launch(h, "layer_rowdot_q", st, [&] { return gas::launch_layer_rowdot(tab, a, st); });
+    ++launches;
+    if (e != cudaSuccess) break;
+    a.which = 0;  // v' = W^K SumGroups(y)
+    a.src = h->ly;
+    a.src_stride = Rq;
+    a.out = h->lv;
+    a.out_stride = s.d;
+    e = launch(h, "layer_coldot_k", st, [&] { return gas::launch_layer_coldot(tab, a, st); });
+    ++launches;
+  }
+  if (e == cudaSuccess) {
+    gas::LayerArgs f{};
+    f.s = s;
+    f.src = h->lu;
+    f.vsrc = h->lv;
+    f.v_out = v_out;
+    f.sigma = sigma;
+    f.scale_out = s_out;
+    f.scale_c = scale_c;
+    f.status = h->status;
+    e = launch(h, "layer_finalize", st, [&] { return gas::launch_layer_finalize(f, st); });
+    ++launches;
+  }
+  h->last_launches = launches;
+  if (e != cudaSuccess) return cuda_fail(h, e, "whole-layer launch");
+  return GAS_OK;
+}
+
 gas_status resolve(gas_ctx* h, double gamma, double delta_star, double r_max, double* g_out, double* a_out) {
   if (!(delta_star > 0.0)) return fail(h, GAS_ERR_INVALID_ARG, "delta_star must be > 0");
   if (!(r_max > 0.0)) return fail(h, GAS_ERR_INVALID_ARG, "r_max must be > 0");
@@ -405,6 +468,10 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_y = take(L * NQ * DH * 4);
   const size_t o_maps = take((2 * L + 1) * sizeof(CUtensorMap));
   const size_t o_flags = take(L * s.tiles_k * sizeof(unsigned));
+  const size_t o_lz = take(L * static_cast<size_t>(n_kv) * d_h * 4);
+  const size_t o_lu = take(L * static_cast<size_t>(d) * 4);
+  const size_t o_ly = take(L * static_cast<size_t>(n_q) * d_h * 4);
+  const size_t o_lv = take(L * static_cast<size_t>(d) * 4);
   h->ws_bytes = off;
   e = cudaMalloc(&h->ws, h->ws_bytes);
   if (e != cudaSuccess) {
@@ -425,6 +492,10 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   h->ybuf = reinterpret_cast<float*>(b + o_y);
   h->dmaps = reinterpret_cast<CUtensorMap*>(b + o_maps);
   h->flags = reinterpret_cast<unsigned*>(b + o_flags);
+  h->lz = reinterpret_cast<float*>(b + o_lz);
+  h->lu = reinterpret_cast<float*>(b + o_lu);
+  h->ly = reinterpret_cast<float*>(b + o_ly);
+  h->lv = reinterpret_cast<float*>(b + o_lv);
   h->hmaps.assign(2 * L + 1, CUtensorMap{});
   h->map_q.assign(L, nullptr);
   h->map_k.assign(L, nullptr);
@@ -506,6 +577,37 @@ gas_status gas_refresh(gas_handle h, const void* const* wq, const void* const* w
   gas_status gs = resolve(h, gamma, delta_star, r_max, &g, &a);
   if (gs != GAS_OK) return gs;
   return spectral_impl(h, wq, wk, iters, v_in, v_out, sigma, s, scale_constant(h, a, r_max), stream);
+}
+
+gas_status gas_layer_refresh(gas_handle h, const void* const* wq, const void* const* wk, int iters,
+                             const float* v_in, float* v_out, float* sigma, double gamma, double delta_star,
+                             double r_max, float* s, void* stream) {
+  if (!h) return GAS_ERR_INVALID_ARG;
+  if (iters < 1) return fail(h, GAS_ERR_INVALID_ARG, "iters must be >= 1 (got %d)", iters);
+  gas_status gs = check_weights(h, wq, wk);
+  if (gs != GAS_OK) return gs;
+  if (!v_in || !sigma) return fail(h, GAS_ERR_INVALID_ARG, "v_in and sigma must not be NULL");
+  if (!aligned16(v_in) || (v_out && !aligned16(v_out)))
+    return fail(h, GAS_ERR_INVALID_ARG, "v_in / v_out must be 16-byte aligned");
+  if (static_cast<size_t>(h->s.d + 8) * 4 > 227 * 1024 ||
+      static_cast<size_t>(h->s.nq * h->s.dh + 2048) * 4 > 227 * 1024)
+    return fail(h, GAS_ERR_UNSUPPORTED, "whole-layer path keeps a d- or n_q*d_h-vector in shared memory");
+  float c = 0.0f;
+  if (s) {
+    double g, a;
+    gs = resolve(h, gamma, delta_star, r_max, &g, &a);
+    if (gs != GAS_OK) return gs;
+    c = scale_constant(h, a, r_max);
+  }
+  cudaError_t e = cudaSetDevice(h->device);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaSetDevice");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  h->last_stream = st;
+  h->launch_names.clear();
+  gas::LayerTable tab;
+  std::memset(&tab, 0, sizeof(tab));
+  fill_table(h, tab, wq, wk);
+  return run_layer(h, tab, iters, v_in, v_out, sigma, s, c, st);
 }
 
 double gas_gamma_min(int d_h, long long n_heads_total, int seq_len, double delta_star) {

@@ -120,13 +120,32 @@ __device__ __forceinline__ TileRef decode_tile(const Shape& s, int t) {
 // of a query tile's G_Q at a time from the row-per-thread layout tcgen05.ld produces to
 // the block layout of the iteration; xs / ts hold the current x and t' of each head
 // slot (two heads per tile when d_h = 64); red the per-warp partial dot products.
+// Layout of a 4-float chunk q of a 128-float row inside a "plane" array: chunks that the
+// lanes of a half-warp read together (same plane, consecutive q / 2 ... see plane_off)
+// are contiguous, so 128-bit shared loads and stores are free of bank conflicts.
 struct EpiSmem {
-  float stage[32][129];
-  float xs[2][128];
-  float ts[2][128];
-  float red[2][2][8];  // [slot][which dot][warp of the head group]
+  float stage[2][32][68];  // [plane][row][16 chunks x 4 floats + 4 pad]
+  float xs[2][2][64];      // [slot][plane][64]: x in the same plane layout
+  float ts[2][2][64];
+  float red[2][2][8];      // [slot][which dot][warp of the head group]
   int ok[2];
 };
+
+// Column col (of a d_h-wide row) -> offset inside [plane][16 chunks][4] when each thread
+// owns cpt consecutive columns (cpt = 8: two planes, cpt = 4: one plane).
+template <int CPT>
+__device__ __forceinline__ int plane_off(int col, int row_stride) {
+  const int p = (CPT == 8) ? ((col >> 2) & 1) : 0;
+  const int slot = col / CPT;
+  return p * 32 * row_stride + slot * 4 + (col & 3);
+}
+
+// The same layout for a single d_h-vector: [plane][16 chunks x 4].
+template <int CPT>
+__device__ __forceinline__ int vec_off(int col) {
+  const int p = (CPT == 8) ? ((col >> 2) & 1) : 0;
+  return p * 64 + (col / CPT) * 4 + (col & 3);
+}
 
 // Sum over the 16 lanes of a half-warp of 8 values per lane: on return v[0] holds the
 // total of value number `idx` (3 halving exchange steps plus one butterfly step).
@@ -193,11 +212,14 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
   const int cb = CPT * cg;                        // first of my columns
   const int myq = (hs * DH + rb) >> 5;            // lane quarter holding my rows
   float gq[8][CPT];
+  float* stage = &ep->stage[0][0][0];
 #pragma unroll 1
   for (int qq = 0; qq < 4; ++qq) {
     if (q == qq) {
 #pragma unroll
-      for (int c = 0; c < HALF; ++c) ep->stage[lane][half * HALF + c] = rowv[c];
+      for (int c = 0; c < HALF; c += 4)
+        *reinterpret_cast<float4*>(stage + lane * 68 + plane_off<CPT>(half * HALF + c, 68)) =
+            make_float4(rowv[c], rowv[c + 1], rowv[c + 2], rowv[c + 3]);
     }
     named_bar_sync(5, 256);
     if (myq == qq) {
@@ -205,7 +227,10 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
 #pragma unroll
       for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int k = 0; k < CPT; ++k) gq[i][k] = ep->stage[r0 + i][cb + k];
+        for (int k = 0; k < CPT; k += 4) {
+          const float4 g4 = *reinterpret_cast<const float4*>(stage + (r0 + i) * 68 + plane_off<CPT>(cb + k, 68));
+          gq[i][k] = g4.x; gq[i][k + 1] = g4.y; gq[i][k + 2] = g4.z; gq[i][k + 3] = g4.w;
+        }
     }
     named_bar_sync(5, 256);
   }
@@ -232,9 +257,11 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
     gk[4][k] = a1.x; gk[5][k] = a1.y; gk[6][k] = a1.z; gk[7][k] = a1.w;
   }
   const size_t hidx = static_cast<size_t>(layer) * s.nq + head;
-  float* xs = ep->xs[hs];
-  float* ts = ep->ts[hs];
-  if (th < DH) xs[th] = __ldcg(a.z0 + (hidx * 2) * DH + th) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + th);
+  // x and t' live in the plane layout (row stride 0: one "row" per slot).
+  float* xs = &ep->xs[hs][0][0];
+  float* ts = &ep->ts[hs][0][0];
+  if (th < DH)
+    xs[vec_off<CPT>(th)] = __ldcg(a.z0 + (hidx * 2) * DH + th) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + th);
   named_bar_sync(bar, NTH);
   const bool writer = (lane & 1) == 0;            // one of the two lanes holding a row total
   float c = 1.0f, sigma = 0.0f, y = 0.0f, n = 0.0f;
@@ -244,7 +271,7 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
     float xv[CPT];
 #pragma unroll
     for (int k = 0; k < CPT; k += 4) {
-      const float4 x4 = *reinterpret_cast<const float4*>(xs + cb + k);
+      const float4 x4 = *reinterpret_cast<const float4*>(xs + vec_off<CPT>(cb + k));
       xv[k] = x4.x; xv[k + 1] = x4.y; xv[k + 2] = x4.z; xv[k + 3] = x4.w;
     }
     float part[8];
@@ -257,8 +284,8 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
     }
     const float tp = halfwarp_transpose_reduce8(part, lane, ridx);
     const int row = rb + ridx;
-    const float xr = xs[row];
-    if (writer) ts[row] = tp;
+    const float xr = xs[vec_off<CPT>(row)];
+    if (writer) ts[vec_off<CPT>(row)] = tp;
     float p = warp_sum(writer ? xr * tp : 0.0f);
     if (lane == 0) ep->red[hs][0][ewh] = p;
     named_bar_sync(bar, NTH);
@@ -273,7 +300,7 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
     // w = G_K y with y = t' / sqrt(S1);  S2 = y . w;  next x = w
 #pragma unroll
     for (int k = 0; k < CPT; k += 4) {
-      const float4 t4 = *reinterpret_cast<const float4*>(ts + cb + k);
+      const float4 t4 = *reinterpret_cast<const float4*>(ts + vec_off<CPT>(cb + k));
       xv[k] = t4.x; xv[k + 1] = t4.y; xv[k + 2] = t4.z; xv[k + 3] = t4.w;
     }
 #pragma unroll
@@ -285,7 +312,7 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
     }
     const float wrow = halfwarp_transpose_reduce8(part, lane, ridx) * inv1;
     y = tp * inv1;
-    if (writer) xs[row] = wrow;
+    if (writer) xs[vec_off<CPT>(row)] = wrow;
     p = warp_sum(writer ? y * wrow : 0.0f);
     if (lane == 0) ep->red[hs][1][ewh] = p;
     named_bar_sync(bar, NTH);

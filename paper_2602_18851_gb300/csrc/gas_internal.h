@@ -118,6 +118,22 @@ struct IterArgs {
   unsigned* status;
 };
 
+// Whole-layer power iteration (Algorithms 2-3 with M = W^Q W^K_exp^T over all heads).
+struct LayerArgs {
+  Shape s;
+  int which;              // 0: key matrix Wk, 1: query matrix Wq
+  const float* src;       // input vector per layer
+  size_t src_stride;      // floats between layers of src (coldot)
+  float* out;
+  size_t out_stride;
+  const float* vsrc;      // finalize: v' of the last iteration
+  float* v_out;           // finalize: [L][d] or null
+  float* sigma;           // finalize: [L]
+  float* scale_out;       // finalize: [L] or null
+  float scale_c;
+  unsigned* status;
+};
+
 struct ScalesArgs {
   int L, nq;
   const float* sigma;
@@ -133,6 +149,9 @@ cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st);
 cudaError_t launch_gram(const GramArgs& a, int num_sms, bool fused, cudaStream_t st);
 cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st);
 cudaError_t launch_writeback(const WbArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_layer_rowdot(const LayerTable& tab, const LayerArgs& a, cudaStream_t st);
+cudaError_t launch_layer_coldot(const LayerTable& tab, const LayerArgs& a, cudaStream_t st);
+cudaError_t launch_layer_finalize(const LayerArgs& a, cudaStream_t st);
 void set_global_error(const char* msg);  // message returned by gas_last_error(NULL)
 size_t gram_smem_bytes(int nz);
 

@@ -1,0 +1,216 @@
+// Whole-layer spectral norm: Algorithms 2-3 (Appendix E) exactly as printed, with one
+// persistent v per layer and M = W^Q W^K_exp^T summed over all heads (Section 4.2):
+//
+//   z_kv = W^K^T v           rowdot over Wk          (n_kv*d_h values)
+//   u'   = W^Q RepeatBlocks(z_kv)   coldot over Wq    (d values)
+//   y    = W^Q^T (u'/||u'||)  rowdot over Wq          (n_q*d_h values)
+//   v'   = W^K SumGroups(y)   coldot over Wk          (d values)
+//
+// In the nn.Linear layout Wq[r][c] (r < n_q*d_h, c < d) is W^Q[c][r], so W^Q^T x is a row
+// dot product and W^Q z a column sum.  The z-space has n_q*d_h dimensions, too many for
+// the d_h x d_h Gram reduction of the per-head path, so every iteration streams each
+// matrix twice.  Normalisations are recomputed by the consumer of a vector from the
+// full vector (d floats), so no partial norms have to travel between kernels.
+
+#include "gas_device.cuh"
+
+namespace gas {
+
+namespace {
+
+constexpr int kRowBlock = 64;  // rows per rowdot CTA (8 warps x 8 rows)
+
+// Stage src[0..n) * (1/||src||) (or * 1 when normalise == 0) into shared memory.
+__device__ __forceinline__ void stage_vector(float* xs, const float* src, int n, int normalise, float* red) {
+  float n2 = 0.0f;
+  if (normalise) {
+    for (int i = threadIdx.x * 4; i < n; i += blockDim.x * 4) {
+      const float4 v = *reinterpret_cast<const float4*>(src + i);
+      n2 = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, n2))));
+    }
+    n2 = warp_sum(n2);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = n2;
+    __syncthreads();
+    n2 = 0.0f;
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) n2 += red[w];
+  }
+  const float inv = normalise ? safe_inv_sqrt(n2) : 1.0f;
+  for (int i = threadIdx.x * 4; i < n; i += blockDim.x * 4) {
+    float4 v = *reinterpret_cast<const float4*>(src + i);
+    v.x *= inv; v.y *= inv; v.z *= inv; v.w *= inv;
+    *reinterpret_cast<float4*>(xs + i) = v;
+  }
+  __syncthreads();
+}
+
+// out[l][r] = sum_c W_l[r][c] * x_l[c] for a block of 64 rows; x = src/||src|| (d values).
+__global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant__ LayerTable tab,
+                                                           const __grid_constant__ LayerArgs a) {
+  extern __shared__ float lsm[];
+  float* xs = lsm;            // [d]
+  float* red = lsm + a.s.d;   // [8]
+  const int l = blockIdx.y;
+  const bool isq = a.which == 1;
+  const int R = (isq ? a.s.nq : a.s.nkv) * a.s.dh;
+  const uint16_t* W = isq ? tab.q[l] : tab.k[l];
+  stage_vector(xs, a.src + static_cast<size_t>(l) * a.s.d, a.s.d, 1, red);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r0 = blockIdx.x * kRowBlock + warp * 8;
+  float acc[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) acc[i] = 0.0f;
+  for (int c = lane * 8; c < a.s.d; c += 256) {
+    const float4 x0 = *reinterpret_cast<const float4*>(xs + c);
+    const float4 x1 = *reinterpret_cast<const float4*>(xs + c + 4);
+    const float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if (r0 + i < R) {
+        const uint4 q = __ldcs(reinterpret_cast<const uint4*>(W + static_cast<size_t>(r0 + i) * a.s.d + c));
+        float f[8];
+        unpack8(q, f);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[i] = fmaf(f[e], xv[e], acc[i]);
+      }
+    }
+  }
+  int idx;
+  const float tot = warp_transpose_reduce<8>(acc, lane, idx);
+  if (transpose_reduce_writer<8>(lane) && r0 + idx < R)
+    a.out[static_cast<size_t>(l) * a.out_stride + r0 + idx] = tot;
+}
+
+// out[l][c] = sum_r W_l[r][c] * x_l[r] for a chunk of 256 columns over all rows, with
+// x = RepeatBlocks(src) (query matrix) or SumGroups(src) (key matrix).
+__global__ void __launch_bounds__(256) layer_coldot_kernel(const __grid_constant__ LayerTable tab,
+                                                           const __grid_constant__ LayerArgs a) {
+  extern __shared__ float lsm[];
+  const Shape& s = a.s;
+  const int l = blockIdx.y;
+  const bool isq = a.which == 1;
+  const int R = (isq ? s.nq : s.nkv) * s.dh;
+  const uint16_t* W = isq ? tab.q[l] : tab.k[l];
+  float* xs = lsm;                  // [R]
+  float* red = lsm + R;             // [8][256]
+  const float* src = a.src + static_cast<size_t>(l) * a.src_stride;
+  for (int r = threadIdx.x; r < R; r += blockDim.x) {
+    const int i = r % s.dh;
+    if (isq) {  // RepeatBlocks(z_kv, G): query row block h reads key block h / G
+      const int hq = r / s.dh;
+      xs[r] = src[(hq / s.G) * s.dh + i];
+    } else {    // SumGroups(y, G): key row block g sums query blocks g*G .. g*G+G-1
+      const int g = r / s.dh;
+      float acc = 0.0f;
+      for (int j = 0; j < s.G; ++j) acc += src[(g * s.G + j) * s.dh + i];
+      xs[r] = acc;
+    }
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x * 256 + lane * 8;
+  float acc[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
+  if (c < s.d) {
+#pragma unroll 4
+    for (int r = warp; r < R; r += 8) {
+      const uint4 q = __ldcs(reinterpret_cast<const uint4*>(W + static_cast<size_t>(r) * s.d + c));
+      float f[8];
+      unpack8(q, f);
+      const float xr = xs[r];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] = fmaf(f[e], xr, acc[e]);
+    }
+  }
+  float4* rp = reinterpret_cast<float4*>(&red[warp * 256 + lane * 8]);
+  rp[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  rp[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+  __syncthreads();
+  const int cc = blockIdx.x * 256 + threadIdx.x;
+  if (cc < s.d) {
+    float tot = 0.0f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) tot += red[w * 256 + threadIdx.x];
+    a.out[static_cast<size_t>(l) * a.out_stride + cc] = tot;
+  }
+}
+
+// sigma_l = ||u'_l|| of the last iteration; v_out = v'/||v'||; fused scale (Eq. 15).
+__global__ void __launch_bounds__(256) layer_finalize_kernel(const __grid_constant__ LayerArgs a) {
+  __shared__ float red[8];
+  const Shape& s = a.s;
+  const int l = blockIdx.x;
+  const float* u = a.src + static_cast<size_t>(l) * s.d;
+  float n2 = 0.0f;
+  for (int i = threadIdx.x * 4; i < s.d; i += blockDim.x * 4) {
+    const float4 v = *reinterpret_cast<const float4*>(u + i);
+    n2 = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, n2))));
+  }
+  n2 = warp_sum(n2);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = n2;
+  __syncthreads();
+  float tot = 0.0f;
+  for (int w = 0; w < 8; ++w) tot += red[w];
+  const float sigma = sqrtf(tot);
+  if (a.v_out != nullptr) {
+    __syncthreads();
+    const float* vp = a.vsrc + static_cast<size_t>(l) * s.d;
+    float m2 = 0.0f;
+    for (int i = threadIdx.x * 4; i < s.d; i += blockDim.x * 4) {
+      const float4 v = *reinterpret_cast<const float4*>(vp + i);
+      m2 = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, m2))));
+    }
+    m2 = warp_sum(m2);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m2;
+    __syncthreads();
+    float mt = 0.0f;
+    for (int w = 0; w < 8; ++w) mt += red[w];
+    const float inv = safe_inv_sqrt(mt);
+    float* vo = a.v_out + static_cast<size_t>(l) * s.d;
+    for (int i = threadIdx.x * 4; i < s.d; i += blockDim.x * 4) {
+      float4 v = *reinterpret_cast<const float4*>(vp + i);
+      v.x *= inv; v.y *= inv; v.z *= inv; v.w *= inv;
+      *reinterpret_cast<float4*>(vo + i) = v;
+    }
+  }
+  if (threadIdx.x == 0) {
+    a.sigma[l] = sigma;
+    if (!isfinite(sigma)) set_status(a.status, GAS_DEV_NONFINITE_SIGMA);
+    if (a.scale_out != nullptr) a.scale_out[l] = a.scale_c * sigma;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_layer_rowdot(const LayerTable& tab, const LayerArgs& a, cudaStream_t st) {
+  const int R = (a.which == 1 ? a.s.nq : a.s.nkv) * a.s.dh;
+  const dim3 grid((R + kRowBlock - 1) / kRowBlock, a.s.L);
+  const size_t smem = (a.s.d + 8) * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(layer_rowdot_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  layer_rowdot_kernel<<<grid, 256, smem, st>>>(tab, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_layer_coldot(const LayerTable& tab, const LayerArgs& a, cudaStream_t st) {
+  const int R = (a.which == 1 ? a.s.nq : a.s.nkv) * a.s.dh;
+  const dim3 grid((a.s.d + 255) / 256, a.s.L);
+  const size_t smem = (R + 8 * 256) * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(layer_coldot_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  layer_coldot_kernel<<<grid, 256, smem, st>>>(tab, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_layer_finalize(const LayerArgs& a, cudaStream_t st) {
+  layer_finalize_kernel<<<a.s.L, 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace gas
