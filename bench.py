@@ -254,6 +254,9 @@ def main():
     rank, world, local = init_dist(args)
     if args.impl == "reference":
         run_reference(args, rank, world)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
         return
     import paper_2602_18851_gb300 as gas
 
