@@ -11,6 +11,9 @@ Pieces (each cites the passage it restates):
   ``mode="factored"``); Algorithm 3 (Appendix E.2) for a whole layer with
   RepeatBlocks / SumGroups, and the explicit W^K expansion it avoids.
 * ``calib.py`` — Eq. 12 (gamma), Eq. 13 (alpha_min), Eq. 15 (per-layer scale).
+* ``fp8.py`` — the consumer of the scale: E4M3 cast of S / scale with overflow
+  statistics (Algorithm 1, Stage 3; Table 4), delayed scaling (Eq. 1) and auto-alpha
+  (Section 3.5, Eq. 16, Algorithm 4).
 
 Readings where the paper is silent: sigma is the last iteration's ||M v_{k-1}||;
 a zero start vector or a zero sigma gives sigma = 0 and v_out = 0; head h uses KV
