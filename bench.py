@@ -7,7 +7,11 @@ per-layer E4M3 scales, with the v write-back.  Inputs (12.08 GB of bf16 weights)
 are resident in HBM and larger than L2, so no L2 flush is needed between steps.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload NAME] [--method auto|gram|stream]
+                    [--workload NAME] [--method auto|gram|stream] [--path refresh|e4m3]
+
+--path e4m3 measures the scale's consumer instead: one gas_fp8_quantize call (Algorithm
+1, Stage 3) on one Llama-2-70B layer's logits at batch 2 x seq 1024 (2 x 64 x 1024 x
+1024 bf16, 268 MB > L2), cast to E4M3 with its overflow statistics.
 
 Prints one JSON line on rank 0.  Under torchrun every rank refreshes its own replica
 (weak scaling, no collective on the data path); timing is the max over ranks.
@@ -32,6 +36,7 @@ if ROOT not in sys.path:
 from synth import get_workload, make_start_vectors, make_weights  # noqa: E402
 
 METRIC = "full-model sigma+scale refresh ms (Llama-2-70B GQA shape); % of HBM roofline"
+METRIC_E4M3 = "E4M3 cast of one Llama-2-70B layer's attention logits (2x64x1024x1024 bf16) ms; % of HBM roofline"
 
 
 def parse():
@@ -47,6 +52,7 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU-baseline sample budget")
+    p.add_argument("--path", default="refresh", choices=["refresh", "e4m3"])
     return p.parse_args()
 
 
@@ -217,6 +223,145 @@ def oracle_sample_ms(wl, iters, budget_s, wq=None, wk=None, v_in=None):
                       f"extrapolated linearly to all {wl.heads} heads"}
 
 
+def e4m3_logits_shape():
+    """Table 8: Llama-2-70B at batch 2 x sequence 1024; 64 query heads."""
+    return (2, 64, 1024, 1024)
+
+
+def e4m3_inputs(device):
+    """One Llama-2-70B layer's logits S = Q K^T / sqrt(d_h) for tokens on the sqrt(d)
+    sphere (synthetic weights of layer 0) and the scale the library derives for it."""
+    import paper_2602_18851_gb300 as gas
+    from synth.gen import _draw_layer
+    from synth.logits import attention_logits, sphere_tokens
+    wl = get_workload("llama2-70b-gqa")
+    q, k, _ = _draw_layer(wl, 0, device, wl.seed)
+    wq, wk = q.to(torch.bfloat16).contiguous(), k.to(torch.bfloat16).contiguous()
+    b, _, t, _ = e4m3_logits_shape()
+    x = sphere_tokens(b, t, wl.d, wl.seed + 99, device=device)
+    S = attention_logits(wq, wk, wl.n_q, wl.n_kv, wl.d_h, x)
+    del x
+    # the geometry-aware scale of this layer (Eq. 15) with the whole model's alpha_min
+    n_heads = wl.layers * wl.n_q
+    alpha = gas.alpha_min(gas.gamma_min(wl.d_h, n_heads), wl.d, wl.d_h, n_heads)
+    h = gas.Handle(1, wl.d, wl.n_q, wl.n_kv, wl.d_h)
+    h.set_calibration(alpha_override=alpha)
+    v = make_start_vectors(wl.scaled(layers=1), device=device)
+    _, scale, _ = h.refresh([wq], [wk], wl.iters, v, write_back=False)
+    torch.cuda.synchronize(device)
+    h.close()
+    return S, scale
+
+
+def oracle_e4m3_ms(S, scale, budget_s):
+    """The oracle's E4M3 cast on leading chunks of S until about `budget_s` seconds;
+    extrapolated to all of S."""
+    import oracle.fp8 as ofp8
+    flat = S.reshape(-1)
+    sc = np.float32(float(scale.reshape(-1)[0]))
+    chunk = 1 << 22
+    spent, done = 0.0, 0
+    while done < flat.numel() and (spent < budget_s or done == 0):
+        part = flat[done:done + chunk].float().cpu().numpy()
+        t0 = time.perf_counter()
+        ofp8.quantize(part, sc, True)
+        spent += time.perf_counter() - t0
+        done += part.size
+    ms = spent / done * flat.numel() * 1e3
+    return {"value": ms, "unit": "ms", "cores": 1, "kind": "oracle",
+            "sample": f"{done} of {flat.numel()} logits ({100.0 * done / flat.numel():.1f}%), numpy E4M3 "
+                      f"cast with statistics, {spent:.1f} s; extrapolated linearly"}
+
+
+def run_e4m3(args, rank, world, local):
+    import paper_2602_18851_gb300 as gas
+    assert torch.cuda.is_available(), "bench.py needs a CUDA device"
+    dev = torch.device("cuda", local)
+    gas.build()
+    S, scale = e4m3_inputs(dev)
+    n = S.numel()
+    q = torch.empty(S.shape, dtype=torch.uint8, device=dev)
+    stats = gas.fp8_stats_buffer(1, dev)
+    st = gas.Fp8State(80)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        st.quantize(0, S, scale[0:1], q_out=q, stats=stats)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    K = max(1, args.steps)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for k in range(K):
+        evs[k][0].record(stream)
+        step()
+        evs[k][1].record(stream)
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop()
+    ms = max_over_ranks(start.elapsed_time(end) / K, world, dev)
+    kern_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    peak, peak_kind = measured_peaks()
+    algo = 3 * n  # bf16 logits read + one code byte written
+    achieved = algo / (kern_ms * 1e-3) / 1e9
+    info = gas.decode_fp8_stats(stats)[0]
+
+    e2e = None
+    if not args.no_e2e:
+        hs = S.cpu().pin_memory()
+        hq = torch.empty(q.shape, dtype=torch.uint8).pin_memory()
+        hst = torch.empty(stats.shape, dtype=stats.dtype).pin_memory()
+        n_e2e = max(1, min(3, K))
+
+        def e2e_step():
+            S.copy_(hs, non_blocking=True)
+            step()
+            hq.copy_(q, non_blocking=True)
+            hst.copy_(stats, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e = {"value": max_over_ranks(a.elapsed_time(b) / n_e2e, world, dev), "unit": "ms",
+               "h2d_bytes_per_step": int(hs.numel() * hs.element_size()),
+               "d2h_bytes_per_step": int(hq.numel() + hst.numel() * hst.element_size()), "steps": n_e2e}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = oracle_e4m3_ms(S, scale, min(args.cpu_seconds, 10.0))
+    if rank == 0:
+        out = {"metric": METRIC_E4M3, "value": ms, "unit": "ms", "n_gpus": world, "steps": K,
+               "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": False,
+               "scaling": "weak", "vs_baseline": None, "dtype": "bf16 in, f32 divide, e4m3 out",
+               "data": "synthetic",
+               "config": {"workload": "llama2-70b-gqa layer logits", "shape": list(e4m3_logits_shape()),
+                          "elements": n, "scale": float(scale[0]), "saturate": True,
+                          "parallelism": "replicas" if world > 1 else "single-gpu",
+                          "l2": "inputs 268 MB > 129 MB L2, no flush needed"},
+               "roofline": {"bound": "hbm", "kernel": "fp8_quantize", "achieved": achieved, "peak": peak,
+                            "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                            "traffic": None, "algorithmic_bytes": algo, "kernel_ms": kern_ms},
+               "stats": info, "gpu_launches": K, "launches_per_step": 1, "clocks": clk,
+               "e2e": e2e, "cpu_baseline": cpu}
+        print(json.dumps(out), flush=True)
+    st.close()
+
+
 def run_reference(args, rank, world):
     """Reference arm: the oracle as it stands on the host cores, same metric / unit."""
     if rank != 0:
@@ -254,6 +399,12 @@ def main():
     rank, world, local = init_dist(args)
     if args.impl == "reference":
         run_reference(args, rank, world)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+    if args.path == "e4m3":
+        run_e4m3(args, rank, world, local)
         if world > 1:
             import torch.distributed as dist
             dist.destroy_process_group()

@@ -19,6 +19,7 @@ import torch
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libgas.so")
 HEADER = os.path.join(os.path.dirname(HERE), "include", "gas.h")
+HEADERS = [HEADER, os.path.join(os.path.dirname(HERE), "include", "gas_fp8.h")]
 
 GAS_OK = 0
 GAS_ERR_INVALID_ARG = 1
@@ -59,10 +60,13 @@ def build(force: bool = False) -> str:
 
 
 def exported_names() -> List[str]:
-    """Function names declared in include/gas.h."""
-    src = open(HEADER).read()
-    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return re.findall(r"\b(gas_[a-z_]+)\s*\(", src)
+    """Function names declared in include/gas.h and include/gas_fp8.h."""
+    names = []
+    for path in HEADERS:
+        src = open(path).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names += re.findall(r"\b(gas_[a-z0-9_]+)\s*\(", src)
+    return names
 
 
 def load(path: str = LIB_PATH):
@@ -100,6 +104,16 @@ def load(path: str = LIB_PATH):
     lib.gas_last_launch_name.restype = ctypes.c_char_p
     lib.gas_spectral_norms_static.argtypes = [c_int] * 5 + [vp, vp, c_int, vp, vp, vp, vp]
     lib.gas_layer_refresh.argtypes = [vp, vp, vp, c_int, vp, vp, vp, c_double, c_double, c_double, vp, vp]
+    lib.gas_fp8_create.argtypes = [c_int, c_int, c_int, ctypes.POINTER(vp)]
+    lib.gas_fp8_destroy.argtypes = [vp]
+    lib.gas_fp8_reset.argtypes = [vp, ctypes.c_float, vp]
+    lib.gas_fp8_delayed_scales.argtypes = [vp, c_double, vp, vp]
+    lib.gas_fp8_quantize.argtypes = [vp, c_int, vp, c_int, c_ll, vp, vp, c_int, vp, vp]
+    lib.gas_fp8_end_step.argtypes = [vp, vp, c_int, c_int, c_int, vp]
+    lib.gas_fp8_auto_alpha.argtypes = [vp, c_double, c_double, vp, vp]
+    lib.gas_fp8_slack_count.argtypes = [vp, ctypes.POINTER(c_int)]
+    lib.gas_fp8_last_error.argtypes = [vp]
+    lib.gas_fp8_last_error.restype = ctypes.c_char_p
     _lib = lib
     return lib
 
@@ -295,5 +309,116 @@ class Handle:
         return sigma, s, v_out
 
 
-__all__ = ["Handle", "GasError", "load", "build", "gamma_min", "alpha_min", "exported_names",
+GAS_DTYPE_BF16 = 0
+GAS_DTYPE_F32 = 1
+GAS_FP8_SATURATE = 0x1
+GAS_FP8_MAX_SLACK = 16384
+
+
+def _check_fp8(st: int, h=None):
+    if st != GAS_OK:
+        msg = load().gas_fp8_last_error(h)
+        raise GasError(st, (msg or b"").decode())
+
+
+def fp8_stats_buffer(count: int = 1, device=None) -> torch.Tensor:
+    """Device storage for `count` gas_fp8_stats records (24 bytes each)."""
+    return torch.zeros(count, 3, dtype=torch.int64, device=device or "cuda")
+
+
+def decode_fp8_stats(buf: torch.Tensor) -> List[dict]:
+    """Host view of gas_fp8_stats records held in a fp8_stats_buffer tensor."""
+    raw = buf.detach().cpu().contiguous()
+    f = raw.view(torch.float32).view(-1, 6)
+    return [{"amax": float(f[i, 0]), "max_scaled": float(f[i, 1]), "overflow": int(raw[i, 1]),
+             "count": int(raw[i, 2])} for i in range(raw.shape[0])]
+
+
+class Fp8State:
+    """The consumer side of the scales (include/gas_fp8.h): E4M3 cast with overflow
+    statistics (Algorithm 1, Stage 3), delayed-scaling history (Eq. 1) and the auto-alpha
+    slack buffer (Section 3.5, Algorithm 4)."""
+
+    def __init__(self, layers: int, history_len: int = 16, burn_in_steps: int = 0):
+        lib = load()
+        self.layers = layers
+        h = ctypes.c_void_p()
+        _check_fp8(lib.gas_fp8_create(int(layers), int(history_len), int(burn_in_steps), ctypes.byref(h)), None)
+        self._h = h
+
+    def close(self):
+        if getattr(self, "_h", None):
+            load().gas_fp8_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def reset(self, history_init: float = 1.0, stream=None):
+        _check_fp8(load().gas_fp8_reset(self._h, float(history_init), _stream_ptr(stream)), self._h)
+
+    def delayed_scales(self, eta: float = 0.9, out: Optional[torch.Tensor] = None, stream=None):
+        """Eq. 1 for every layer."""
+        if out is None:
+            out = torch.empty(self.layers, device="cuda", dtype=torch.float32)
+        _check_fp8(load().gas_fp8_delayed_scales(self._h, float(eta), out.data_ptr(), _stream_ptr(stream)),
+                   self._h)
+        return out
+
+    def quantize(self, layer: int, s: torch.Tensor, scale: torch.Tensor, q_out: Optional[torch.Tensor] = None,
+                 saturate: bool = True, stats: Optional[torch.Tensor] = None, want_codes: bool = True,
+                 stream=None):
+        """S / scale -> E4M3 codes (uint8, same shape as S) and one stats record.
+        `scale` is a one-element float32 CUDA tensor (e.g. s[l:l+1])."""
+        if s.dtype == torch.bfloat16:
+            dt = GAS_DTYPE_BF16
+        elif s.dtype == torch.float32:
+            dt = GAS_DTYPE_F32
+        else:
+            raise ValueError("logits must be bfloat16 or float32")
+        if not s.is_contiguous() or not s.is_cuda:
+            raise ValueError("logits must be a contiguous CUDA tensor")
+        if scale.dtype != torch.float32 or scale.numel() < 1:
+            raise ValueError("scale must be a float32 CUDA tensor with at least one element")
+        if q_out is None and want_codes:
+            q_out = torch.empty(s.shape, dtype=torch.uint8, device=s.device)
+        if stats is None:
+            stats = fp8_stats_buffer(1, s.device)
+        st = load().gas_fp8_quantize(self._h, int(layer), s.data_ptr() if s.numel() else None, dt, s.numel(),
+                                     scale.data_ptr(), q_out.data_ptr() if q_out is not None else None,
+                                     GAS_FP8_SATURATE if saturate else 0, stats.data_ptr(), _stream_ptr(stream))
+        _check_fp8(st, self._h)
+        return q_out, stats
+
+    def end_step(self, sigma: Optional[torch.Tensor] = None, d: int = 0, d_h: int = 0, stream=None):
+        """Push the step maxima into the history; with sigma ([layers, n_q]) also record
+        the slack ratios of Eq. 16."""
+        n_q = int(sigma.shape[-1]) if sigma is not None else 0
+        _check_fp8(load().gas_fp8_end_step(self._h, sigma.data_ptr() if sigma is not None else None, n_q,
+                                           int(d), int(d_h), _stream_ptr(stream)), self._h)
+
+    def auto_alpha(self, q: float = 0.9999, kappa: float = 1.0, out: Optional[torch.Tensor] = None, stream=None):
+        """Algorithm 4 on the recorded slack ratios (one float32 on the device)."""
+        if out is None:
+            out = torch.empty(1, device="cuda", dtype=torch.float32)
+        _check_fp8(load().gas_fp8_auto_alpha(self._h, float(q), float(kappa), out.data_ptr(), _stream_ptr(stream)),
+                   self._h)
+        return out
+
+    def slack_count(self) -> int:
+        c = ctypes.c_int()
+        _check_fp8(load().gas_fp8_slack_count(self._h, ctypes.byref(c)), self._h)
+        return c.value
+
+
+__all__ = ["Handle", "Fp8State", "fp8_stats_buffer", "decode_fp8_stats", "GasError", "load", "build", "gamma_min", "alpha_min", "exported_names",
            "METHOD_AUTO", "METHOD_STREAM", "METHOD_GRAM", "METHOD_FUSED", "E4M3_MAX", "LIB_PATH"]

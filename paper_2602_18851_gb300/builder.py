@@ -15,7 +15,8 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libgas.so")
 
-SOURCES = ["gas_api.cpp", "gas_stream.cu", "gas_gram.cu", "gas_writeback.cu", "gas_static.cu", "gas_layer.cu"]
+SOURCES = ["gas_api.cpp", "gas_stream.cu", "gas_gram.cu", "gas_writeback.cu", "gas_static.cu", "gas_layer.cu",
+           "gas_fp8.cu"]
 HEADERS = ["gas_device.cuh", "gas_internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
@@ -32,7 +33,7 @@ def _stale() -> bool:
     if not os.path.exists(LIB):
         return True
     t = os.path.getmtime(LIB)
-    deps = [os.path.join(CSRC, f) for f in SOURCES + HEADERS] + [os.path.join(INCLUDE, "gas.h"),
+    deps = [os.path.join(CSRC, f) for f in SOURCES + HEADERS] + [os.path.join(INCLUDE, "gas.h"), os.path.join(INCLUDE, "gas_fp8.h"),
                                                                  os.path.abspath(__file__)]
     return any(os.path.getmtime(p) > t for p in deps)
 
