@@ -63,7 +63,9 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
   constexpr int GPT = 128 / DH;  // groups per key tile
   constexpr uint32_t YB = Cfg::kYBytes;
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  // 1024-byte alignment by pointer arithmetic on the shared array itself, so that the
+  // compiler keeps every derived pointer in the shared address space.
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint8_t* ring = smem;                      // [S][kStage]
   uint8_t* ybuf_s = smem + S * kStage;       // [2][YB]
   uint64_t* bars = reinterpret_cast<uint64_t*>(ybuf_s + 2 * YB);
