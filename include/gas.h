@@ -11,11 +11,13 @@
  * with alpha >= alpha_min from Eq. 13 and the typicality gamma from Eq. 12.
  *
  * Conventions shared by every entry point
- *  - Weights use the nn.Linear layout, bf16, row-major, one allocation per layer:
+ *  - Weights use the nn.Linear layout, bf16, row-major, one pointer per layer:
  *      Wq[l] : [n_q  * d_h, d]   rows h*d_h .. h*d_h+d_h-1 are (W^Q_h)^T
  *      Wk[l] : [n_kv * d_h, d]   rows g*d_h .. are (W^K_g)^T
- *    Query head h uses KV group g(h) = h / (n_q / n_kv) (RepeatBlocks order,
- *    Appendix F).  Each layer pointer must be 16-byte aligned.
+ *    contiguous by default; gas_set_weight_layout describes padded rows and
+ *    per-head-interleaved (fused projection) storage.  Query head h uses KV group
+ *    g(h) = h / (n_q / n_kv) (RepeatBlocks order, Appendix F).  Each layer pointer
+ *    must be 16-byte aligned.
  *  - Vectors are fp32, [layers][n_q][d] contiguous, 16-byte aligned.
  *  - The caller owns every buffer passed in.  The handle owns only its workspace
  *    (device memory sized at gas_create) and cached TMA descriptors.
@@ -155,6 +157,26 @@ double gas_alpha_min(double gamma, int d, int d_h, long long n_heads_total, int 
 /* Gamma and alpha the handle would use for gas_scales with this gamma / delta*. */
 gas_status gas_resolve_calibration(gas_handle h, double gamma, double delta_star,
                                    double *gamma_out, double *alpha_out);
+
+/*
+ * Weight layout (SURVEY row "layout generality"; the paper fixes none).  By default a
+ * layer's Wq[l] is the contiguous nn.Linear matrix [n_q * d_h, d].  Weights that are a
+ * strided view of a larger allocation are described by two strides per matrix, in
+ * elements:
+ *     element (row i of head j, column c) of Wq[l] is at Wq[l][j * hs_q + i * ld_q + c]
+ * (likewise Wk[l] with ld_k, hs_k and key groups j).  This covers rows padded beyond d
+ * (ld > d), and fused projections whose query and key blocks are interleaved per head,
+ * e.g. [heads][3][d_h][d] gives ld = d, hs = 3 * d_h * d with Wk[l] = Wq[l] + d_h * d.
+ *   layout  GAS_LAYOUT_ROWS (the only one implemented; others -> GAS_ERR_UNSUPPORTED)
+ *   ld_q, ld_k  row strides, >= d; 0 = d
+ *   hs_q, hs_k  head strides, >= d_h * row stride (heads do not overlap); 0 = d_h * ld
+ * All strides must be multiples of 8 elements (16-byte rows and heads, as TMA needs).
+ * Host only; applies to every later call on the handle (gas_spectral_norms_static always
+ * uses the contiguous layout).  Errors: GAS_ERR_INVALID_ARG with a message.
+ */
+#define GAS_LAYOUT_ROWS 0
+gas_status gas_set_weight_layout(gas_handle h, int layout, long long ld_q, long long ld_k, long long hs_q,
+                                 long long hs_k);
 
 /* Message for the last error on this handle (or the last gas_create failure when h is NULL). */
 const char *gas_last_error(gas_handle h);

@@ -104,6 +104,7 @@ def load(path: str = LIB_PATH):
     lib.gas_last_launch_name.restype = ctypes.c_char_p
     lib.gas_spectral_norms_static.argtypes = [c_int] * 5 + [vp, vp, c_int, vp, vp, vp, vp]
     lib.gas_layer_refresh.argtypes = [vp, vp, vp, c_int, vp, vp, vp, c_double, c_double, c_double, vp, vp]
+    lib.gas_set_weight_layout.argtypes = [vp, c_int, c_ll, c_ll, c_ll, c_ll]
     lib.gas_fp8_create.argtypes = [c_int, c_int, c_int, ctypes.POINTER(vp)]
     lib.gas_fp8_destroy.argtypes = [vp]
     lib.gas_fp8_reset.argtypes = [vp, ctypes.c_float, vp]
@@ -136,13 +137,24 @@ def alpha_min(gamma: float, d: int, d_h: int, n_heads_total: int, seq_len: int =
                                 float(delta_star))
 
 
-def _ptr_array(tensors: Sequence[torch.Tensor], rows: int, d: int, name: str):
+def _ptr_array(tensors: Sequence[torch.Tensor], rows: int, d: int, name: str, layout=None):
+    """Device pointers of per-layer weight tensors.  Default layout: each tensor is the
+    contiguous [rows, d] matrix.  With a strided layout (heads, d_h, ld, hs) each tensor
+    starts at the matrix's first element and must cover its last one."""
     arr = (ctypes.c_void_p * len(tensors))()
     for i, t in enumerate(tensors):
-        if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
-            raise ValueError(f"{name}[{i}] must be a contiguous CUDA bfloat16 tensor")
-        if tuple(t.shape) != (rows, d):
-            raise ValueError(f"{name}[{i}] has shape {tuple(t.shape)}, expected {(rows, d)}")
+        if t.dtype != torch.bfloat16 or not t.is_cuda:
+            raise ValueError(f"{name}[{i}] must be a CUDA bfloat16 tensor")
+        if layout is None:
+            if not t.is_contiguous() or tuple(t.shape) != (rows, d):
+                raise ValueError(f"{name}[{i}] must be contiguous with shape {(rows, d)}, got {tuple(t.shape)}")
+        else:
+            heads, dh, ld, hs = layout
+            last = (heads - 1) * hs + (dh - 1) * ld + d - 1
+            avail = t.untyped_storage().nbytes() // 2 - t.storage_offset()
+            if last >= avail:
+                raise ValueError(f"{name}[{i}]: the strided matrix needs {last + 1} elements, "
+                                 f"the tensor's storage holds {avail} from its first element")
         arr[i] = t.data_ptr()
     return arr
 
@@ -164,6 +176,7 @@ class Handle:
         h = ctypes.c_void_p()
         _check(lib.gas_create(layers, d, n_q, n_kv, d_h, ctypes.byref(h)), None)
         self._h = h
+        self._lq = self._lk = None  # strided layouts of Wq / Wk (None: contiguous)
 
     # -- lifetime --------------------------------------------------------------------
     def close(self):
@@ -191,6 +204,24 @@ class Handle:
     def set_calibration(self, seq_len: int = 1024, eta_fp8: float = 0.8, alpha_override: float = 0.0):
         _check(load().gas_set_calibration(self._h, int(seq_len), float(eta_fp8), float(alpha_override)),
                self._h)
+
+    def set_weight_layout(self, ld_q: int = 0, ld_k: int = 0, head_stride_q: int = 0, head_stride_k: int = 0):
+        """Strided weights (include/gas.h, gas_set_weight_layout): element (row i of head
+        j, column c) at w[j * head_stride + i * ld + c]; 0 keeps the contiguous default."""
+        _check(load().gas_set_weight_layout(self._h, 0, int(ld_q), int(ld_k), int(head_stride_q),
+                                            int(head_stride_k)), self._h)
+        lq = ld_q or self.d
+        lk = ld_k or self.d
+        hq = head_stride_q or lq * self.d_h
+        hk = head_stride_k or lk * self.d_h
+        default = (lq == self.d and lk == self.d and hq == self.d * self.d_h and hk == self.d * self.d_h)
+        self._lq = None if default else (self.n_q, self.d_h, lq, hq)
+        self._lk = None if default else (self.n_kv, self.d_h, lk, hk)
+
+    def _weights(self, wq, wk):
+        lq, lk = getattr(self, "_lq", None), getattr(self, "_lk", None)
+        return (_ptr_array(wq, self.n_q * self.d_h, self.d, "wq", lq),
+                _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk", lk))
 
     def set_method(self, method):
         m = METHODS[method] if isinstance(method, str) else int(method)
@@ -243,8 +274,7 @@ class Handle:
                        sigma: Optional[torch.Tensor] = None, write_back: bool = True, stream=None):
         """sigma[l,h] after `iters` power iterations from v_in; v_out the unit right
         singular vector estimates (warm start for the next call).  Returns (sigma, v_out)."""
-        qa = _ptr_array(wq, self.n_q * self.d_h, self.d, "wq")
-        ka = _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk")
+        qa, ka = self._weights(wq, wk)
         if v_out is None and write_back:
             v_out = torch.empty_like(v_in)
         v_out, sigma = self._vec_args(v_in, v_out, sigma, v_in.device)
@@ -269,8 +299,7 @@ class Handle:
                 gamma: float = 0.0, delta_star: float = 1e-6, r_max: float = E4M3_MAX,
                 write_back: bool = True, stream=None):
         """Spectral norms and per-layer scales in one call.  Returns (sigma, s, v_out)."""
-        qa = _ptr_array(wq, self.n_q * self.d_h, self.d, "wq")
-        ka = _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk")
+        qa, ka = self._weights(wq, wk)
         if v_out is None and write_back:
             v_out = torch.empty_like(v_in)
         v_out, sigma = self._vec_args(v_in, v_out, sigma, v_in.device)
@@ -290,8 +319,7 @@ class Handle:
                       write_back: bool = True, with_scales: bool = True, stream=None):
         """Whole-layer sigma_l = ||W^Q W^K_exp^T||_2 (Algorithms 2-3 over all heads), one v
         per layer: v_in [layers, d].  Returns (sigma[layers], s[layers] or None, v_out)."""
-        qa = _ptr_array(wq, self.n_q * self.d_h, self.d, "wq")
-        ka = _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk")
+        qa, ka = self._weights(wq, wk)
         shape = (self.layers, self.d)
         if v_in.dtype != torch.float32 or tuple(v_in.shape) != shape or not v_in.is_contiguous():
             raise ValueError(f"v_in must be a contiguous float32 tensor of shape {shape}")

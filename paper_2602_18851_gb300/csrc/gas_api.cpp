@@ -112,6 +112,23 @@ bool encode_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, u
   return r == CUDA_SUCCESS;
 }
 
+// 3D bf16 map of one weight matrix: (column c, row i inside a head, head j) at
+// base + j * hs + i * ld + c; box 64 columns x d_h rows x 128/d_h heads, so a box is one
+// 128-row tile in the canonical K-major SW128 layout whatever the strides.
+bool encode_weights(CUtensorMap* m, const void* base, uint64_t d, uint32_t dh, uint64_t heads, uint64_t ld,
+                    uint64_t hs) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {d, dh, heads};
+  cuuint64_t strides[2] = {ld * 2, hs * 2};
+  cuuint32_t box[3] = {64, dh, 128 / dh};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 float scale_constant(const gas_ctx* h, double alpha, double r_max) {
   return static_cast<float>(alpha * (static_cast<double>(h->s.d) / std::sqrt(static_cast<double>(h->s.dh))) /
                             (h->eta_fp8 * r_max));
@@ -135,8 +152,9 @@ gas_status ensure_maps(gas_ctx* h, const void* const* wq, const void* const* wk,
   for (int l = 0; same && l < L; ++l) same = (h->map_q[l] == wq[l] && h->map_k[l] == wk[l]);
   if (same) return GAS_OK;
   for (int l = 0; l < L; ++l) {
-    if (!encode_2d(&h->hmaps[l], wq[l], h->s.d, static_cast<uint64_t>(h->s.nq) * h->s.dh, 128) ||
-        !encode_2d(&h->hmaps[L + l], wk[l], h->s.d, static_cast<uint64_t>(h->s.nkv) * h->s.dh, 128))
+    const Shape& sh = h->s;
+    if (!encode_weights(&h->hmaps[l], wq[l], sh.d, sh.dh, sh.nq, sh.ldq, sh.hsq) ||
+        !encode_weights(&h->hmaps[L + l], wk[l], sh.d, sh.dh, sh.nkv, sh.ldk, sh.hsk))
       return fail(h, GAS_ERR_CUDA, "cuTensorMapEncodeTiled failed for layer %d", l);
     h->map_q[l] = wq[l];
     h->map_k[l] = wk[l];
@@ -432,6 +450,8 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   s.tiles_k = (n_kv * d_h + 127) / 128;
   s.nkc = (d + 63) / 64;
   s.nz = nz_t;
+  s.ldq = s.ldk = d;
+  s.hsq = s.hsk = static_cast<long long>(d_h) * d;
 
   cudaError_t e = cudaGetDevice(&h->device);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
@@ -542,6 +562,30 @@ gas_status gas_set_method(gas_handle h, int method) {
       method != GAS_METHOD_FUSED)
     return fail(h, GAS_ERR_INVALID_ARG, "unknown method %d", method);
   h->method = method;
+  return GAS_OK;
+}
+
+gas_status gas_set_weight_layout(gas_handle h, int layout, long long ld_q, long long ld_k, long long hs_q,
+                                 long long hs_k) {
+  if (!h) return GAS_ERR_INVALID_ARG;
+  if (layout != GAS_LAYOUT_ROWS)
+    return fail(h, GAS_ERR_UNSUPPORTED, "layout %d is not implemented (only GAS_LAYOUT_ROWS)", layout);
+  const Shape& s = h->s;
+  const long long lq = ld_q ? ld_q : s.d, lk = ld_k ? ld_k : s.d;
+  const long long hq = hs_q ? hs_q : lq * s.dh, hk = hs_k ? hs_k : lk * s.dh;
+  if (lq < s.d || lk < s.d)
+    return fail(h, GAS_ERR_INVALID_ARG, "row strides must be >= d (%d), got %lld and %lld", s.d, lq, lk);
+  if (hq < lq * s.dh || hk < lk * s.dh)
+    return fail(h, GAS_ERR_INVALID_ARG, "head strides must be >= d_h * row stride (heads must not overlap)");
+  if (lq % 8 || lk % 8 || hq % 8 || hk % 8)
+    return fail(h, GAS_ERR_INVALID_ARG, "row and head strides must be multiples of 8 elements (16 bytes)");
+  if ((lq >> 37) || (lk >> 37) || (hq >> 37) || (hk >> 37))
+    return fail(h, GAS_ERR_INVALID_ARG, "strides too large");
+  h->s.ldq = lq;
+  h->s.ldk = lk;
+  h->s.hsq = hq;
+  h->s.hsk = hk;
+  h->maps_valid = false;  // descriptors are rebuilt at the next call
   return GAS_OK;
 }
 

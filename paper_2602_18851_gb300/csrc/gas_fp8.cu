@@ -4,8 +4,9 @@
 //                         per-call statistics of Table 4 (largest scaled logit, number of
 //                         scaled logits beyond 448) and the step maximum max|S| that the
 //                         delayed-scaling history (Eq. 1) and the slack ratio (Eq. 16) use.
-//                         One streaming pass: 16 logits per thread and step (two or four
-//                         16-byte loads, one 16-byte store of codes); per-CTA reductions
+//                         One streaming pass: 16 logits per thread and group (two or four
+//                         16-byte loads, one 16-byte store of codes), four groups (bf16) or
+//                         two (fp32) in flight per thread; per-CTA reductions
 //                         go to a per-layer accumulator by atomics, and the last CTA to
 //                         finish (ticket counter, no waiting) writes the statistics and
 //                         clears the accumulator for the next call.
@@ -84,14 +85,25 @@ __device__ __forceinline__ uint32_t canon_nan4(uint32_t w) {
   return out;
 }
 
-// Load sixteen logits starting at element 16*g; returns their largest |x| as bits
-// (non-negative floats order like their bit patterns; NaN above infinity).
+// Sixteen logits as loaded: two 16-byte words of bf16, or four of fp32.
 template <int DT>
-__device__ __forceinline__ uint32_t load16(const QArgs& a, long long g, float (&x)[16]) {
+struct Raw16 {
+  uint4 w[DT == GAS_DTYPE_BF16 ? 2 : 4];
+};
+
+template <int DT>
+__device__ __forceinline__ void load16(const QArgs& a, long long g, Raw16<DT>& r) {
+  const uint4* p = reinterpret_cast<const uint4*>(a.s) + (DT == GAS_DTYPE_BF16 ? 2 : 4) * g;
+#pragma unroll
+  for (int i = 0; i < (DT == GAS_DTYPE_BF16 ? 2 : 4); ++i) r.w[i] = __ldcs(p + i);
+}
+
+// Widen sixteen loaded logits to fp32; returns their largest |x| as bits (non-negative
+// floats order like their bit patterns; NaN above infinity).
+template <int DT>
+__device__ __forceinline__ uint32_t unpack16(const Raw16<DT>& r, float (&x)[16]) {
   if (DT == GAS_DTYPE_BF16) {
-    const uint4* p = reinterpret_cast<const uint4*>(a.s) + 2 * g;
-    const uint4 u0 = __ldcs(p), u1 = __ldcs(p + 1);
-    const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+    const uint32_t w[8] = {r.w[0].x, r.w[0].y, r.w[0].z, r.w[0].w, r.w[1].x, r.w[1].y, r.w[1].z, r.w[1].w};
     __nv_bfloat162 m = __halves2bfloat162(__ushort_as_bfloat16(0), __ushort_as_bfloat16(0));
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
@@ -103,15 +115,16 @@ __device__ __forceinline__ uint32_t load16(const QArgs& a, long long g, float (&
     const uint32_t mb = *reinterpret_cast<const uint32_t*>(&m);
     return max(mb << 16, mb & 0xFFFF0000u);
   } else {
-    const float4* p = reinterpret_cast<const float4*>(a.s) + 4 * g;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float4 v = __ldcs(p + i);
-      x[4 * i] = v.x; x[4 * i + 1] = v.y; x[4 * i + 2] = v.z; x[4 * i + 3] = v.w;
-    }
     uint32_t m = 0;
 #pragma unroll
-    for (int i = 0; i < 16; ++i) m = max(m, __float_as_uint(x[i]) & 0x7FFFFFFFu);
+    for (int i = 0; i < 4; ++i) {
+      const uint32_t b[4] = {r.w[i].x, r.w[i].y, r.w[i].z, r.w[i].w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        x[4 * i + j] = __uint_as_float(b[j]);
+        m = max(m, b[j] & 0x7FFFFFFFu);
+      }
+    }
     return m;
   }
 }
@@ -161,10 +174,10 @@ __device__ __forceinline__ uint4 encode16_exact(const float (&x)[16], float sc, 
 }
 
 template <int DT, bool SAT>
-__device__ __forceinline__ uint4 quantize16(const QArgs& a, long long g, float sc, float y, uint32_t thr,
-                                            unsigned& ovf, unsigned& amax) {
+__device__ __forceinline__ uint4 quantize16(const Raw16<DT>& r, float sc, float y, uint32_t thr, unsigned& ovf,
+                                            unsigned& amax) {
   float x[16];
-  const uint32_t gm = load16<DT>(a, g, x);
+  const uint32_t gm = unpack16<DT>(r, x);
   amax = max(amax, gm);
   if (gm < thr) return encode16_fast(x, sc, y);
   return encode16_exact<SAT>(x, sc, ovf);
@@ -213,18 +226,23 @@ __device__ __forceinline__ void quantize_body(const QArgs& a, float sc, unsigned
   const long long stride = static_cast<long long>(gridDim.x) * blockDim.x;
   const long long gt = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
   long long g = gt;
-  // two groups in flight per thread
-  for (; g + stride < groups; g += 2 * stride) {
-    const uint4 c0 = quantize16<DT, SAT>(a, g, sc, y, thr, ovf, amax);
-    const uint4 c1 = quantize16<DT, SAT>(a, g + stride, sc, y, thr, ovf, amax);
-    if (a.q) {
-      __stcs(reinterpret_cast<uint4*>(a.q) + g, c0);
-      __stcs(reinterpret_cast<uint4*>(a.q) + g + stride, c1);
+  // U groups in flight per thread: all loads issued before any group is encoded
+  constexpr int U = DT == GAS_DTYPE_BF16 ? 4 : 2;
+  for (; g + (U - 1) * stride < groups; g += U * stride) {
+    Raw16<DT> r[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) load16<DT>(a, g + u * stride, r[u]);
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint4 c = quantize16<DT, SAT>(r[u], sc, y, thr, ovf, amax);
+      if (a.q) __stcs(reinterpret_cast<uint4*>(a.q) + g + u * stride, c);
     }
   }
-  if (g < groups) {
-    const uint4 c0 = quantize16<DT, SAT>(a, g, sc, y, thr, ovf, amax);
-    if (a.q) __stcs(reinterpret_cast<uint4*>(a.q) + g, c0);
+  for (; g < groups; g += stride) {
+    Raw16<DT> r;
+    load16<DT>(a, g, r);
+    const uint4 c = quantize16<DT, SAT>(r, sc, y, thr, ovf, amax);
+    if (a.q) __stcs(reinterpret_cast<uint4*>(a.q) + g, c);
   }
   // ragged tail: the last n % 16 logits, one per thread of the first CTA
   const long long i = (groups << 4) + gt;
@@ -235,7 +253,7 @@ __device__ __forceinline__ void quantize_body(const QArgs& a, float sc, unsigned
 }
 
 template <int DT, bool SAT>
-__global__ void __launch_bounds__(kThreads, 5) fp8_quantize_kernel(const __grid_constant__ QArgs a) {
+__global__ void __launch_bounds__(kThreads, 3) fp8_quantize_kernel(const __grid_constant__ QArgs a) {
   const float sc = *a.scale;
   unsigned ovf = 0, amax = 0;
   quantize_body<DT, SAT>(a, sc, ovf, amax);

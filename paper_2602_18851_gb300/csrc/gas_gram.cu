@@ -395,7 +395,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           const uint32_t sx = smem_u32(smem + st * SB);
           const uint32_t fb = smem_u32(&full[st]);
           mbar_arrive_expect_tx(fb, tr.is_k ? SB : kTileBytes);
-          tma_load_2d(sx, map, fb, kc * 64, row0, pol);
+          tma_load_3d(sx, map, fb, kc * 64, 0, row0 / DH, pol);  // 128/d_h heads of d_h rows
           if (tr.is_k) tma_load_2d(sx + kTileBytes, a.map_v, fb, kc * 64, vrow0, pol);
           ++issued;
         }

@@ -31,7 +31,16 @@ struct Shape {
   int tiles_k;    // ceil(nkv * dh / 128)
   int nkc;        // ceil(d / 64)
   int nz;         // z-accumulator columns of a K tile (multiple of 16)
+  long long ldq;  // elements between consecutive rows of one head of Wq[l] (>= d)
+  long long ldk;  // elements between consecutive rows of one key group of Wk[l] (>= d)
+  long long hsq;  // elements between the first rows of consecutive query heads (>= d_h * ldq)
+  long long hsk;  // elements between the first rows of consecutive key groups (>= d_h * ldk)
 };
+
+// Element offset of row r (head r / d_h, row r % d_h inside it) of a weight matrix.
+__host__ __device__ inline long long weight_row_offset(int r, int dh, long long ld, long long hs) {
+  return static_cast<long long>(r / dh) * hs + static_cast<long long>(r % dh) * ld;
+}
 
 // ---- streaming matvec-chain passes (Algorithm 2 applied literally) ---------------
 // One pass streams one weight matrix X (a head's A_h or a group's B_g, d_h x d) in

@@ -53,6 +53,8 @@ __global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant
   const bool isq = a.which == 1;
   const int R = (isq ? a.s.nq : a.s.nkv) * a.s.dh;
   const uint16_t* W = isq ? tab.q[l] : tab.k[l];
+  const long long ld = isq ? a.s.ldq : a.s.ldk;
+  const long long hstride = isq ? a.s.hsq : a.s.hsk;
   stage_vector(xs, a.src + static_cast<size_t>(l) * a.s.d, a.s.d, 1, red);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r0 = blockIdx.x * kRowBlock + warp * 8;
@@ -66,7 +68,8 @@ __global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       if (r0 + i < R) {
-        const uint4 q = __ldcs(reinterpret_cast<const uint4*>(W + static_cast<size_t>(r0 + i) * a.s.d + c));
+        const uint4 q =
+            __ldcs(reinterpret_cast<const uint4*>(W + weight_row_offset(r0 + i, a.s.dh, ld, hstride) + c));
         float f[8];
         unpack8(q, f);
 #pragma unroll
@@ -90,6 +93,8 @@ __global__ void __launch_bounds__(256) layer_coldot_kernel(const __grid_constant
   const bool isq = a.which == 1;
   const int R = (isq ? s.nq : s.nkv) * s.dh;
   const uint16_t* W = isq ? tab.q[l] : tab.k[l];
+  const long long ld = isq ? s.ldq : s.ldk;
+  const long long hstride = isq ? s.hsq : s.hsk;
   float* xs = lsm;                  // [R]
   float* red = lsm + R;             // [8][256]
   const float* src = a.src + static_cast<size_t>(l) * a.src_stride;
@@ -114,7 +119,7 @@ __global__ void __launch_bounds__(256) layer_coldot_kernel(const __grid_constant
   if (c < s.d) {
 #pragma unroll 4
     for (int r = warp; r < R; r += 8) {
-      const uint4 q = __ldcs(reinterpret_cast<const uint4*>(W + static_cast<size_t>(r) * s.d + c));
+      const uint4 q = __ldcs(reinterpret_cast<const uint4*>(W + weight_row_offset(r, s.dh, ld, hstride) + c));
       float f[8];
       unpack8(q, f);
       const float xr = xs[r];

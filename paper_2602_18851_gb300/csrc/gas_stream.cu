@@ -30,13 +30,15 @@ __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant_
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int col = chunk * kStreamChunk + lane * 8;
   const bool colok = col < s.d;  // d % 8 == 0: a lane's 8 columns are all in or all out
-  const uint16_t* X = ((MODE == kPassQ) ? tab.q[l] : tab.k[l]) + static_cast<size_t>(m) * DH * s.d;
+  const long long ld = (MODE == kPassQ) ? s.ldq : s.ldk;
+  const long long hstride = (MODE == kPassQ) ? s.hsq : s.hsk;
+  const uint16_t* X = ((MODE == kPassQ) ? tab.q[l] : tab.k[l]) + static_cast<size_t>(m) * hstride;
 
   uint4 w[R];
 #pragma unroll
   for (int rr = 0; rr < R; ++rr) {
     const int row = warp + 8 * rr;
-    w[rr] = colok ? load_stream16(X + static_cast<size_t>(row) * s.d + col) : make_uint4(0, 0, 0, 0);
+    w[rr] = colok ? load_stream16(X + static_cast<size_t>(row) * ld + col) : make_uint4(0, 0, 0, 0);
   }
 
   __shared__ float xs[DH];

@@ -127,8 +127,8 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           const uint32_t fb = smem_u32(&full[st]);
           const uint32_t dst = smem_u32(ring + st * kStage);
           mbar_arrive_expect_tx(fb, kStage);
-          tma_load_2d(dst, &a.maps_k[w.layer], fb, w.c0 + 128 * j, w.tile * 128, pol);
-          tma_load_2d(dst + kBox, &a.maps_k[w.layer], fb, w.c0 + 128 * j + 64, w.tile * 128, pol);
+          tma_load_3d(dst, &a.maps_k[w.layer], fb, w.c0 + 128 * j, 0, w.tile * (128 / DH), pol);
+          tma_load_3d(dst + kBox, &a.maps_k[w.layer], fb, w.c0 + 128 * j + 64, 0, w.tile * (128 / DH), pol);
           ++issued;
         }
       }
