@@ -51,6 +51,10 @@ def _load():
                                                                        ctypes.c_int, dp, dp]
         lib.oracle_layer_form_expanded.argtypes = [ctypes.c_int] * 4 + [u16p, u16p, dp]
         lib.oracle_max_threads.restype = ctypes.c_int
+        lib.oracle_set_weight_format.argtypes = [ctypes.c_int]
+        lib.oracle_set_weight_format.restype = None
+        lib.oracle_decode_weights.argtypes = [u16p, ctypes.c_long, dp]
+        lib.oracle_decode_weights.restype = None
         _lib = lib
     return _lib
 
@@ -104,6 +108,20 @@ def power_iteration_factored(A_bits, B_bits, v0, iters):
     _load().oracle_power_iteration_factored(d, dh, pa, pb, pv, int(iters), ctypes.byref(sig),
                                             v.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
     return sig.value, v
+
+
+def set_weight_format(fmt: str) -> None:
+    """Weight bit format every later call decodes: "bf16" (default) or "f16"."""
+    _load().oracle_set_weight_format({"bf16": 0, "f16": 1}[fmt])
+
+
+def decode_weights(bits) -> np.ndarray:
+    """The oracle's exact float64 value of each 16-bit weight in the current format."""
+    b = np.ascontiguousarray(bits, dtype=np.uint16).ravel()
+    out = np.empty(b.size, dtype=np.float64)
+    _load().oracle_decode_weights(b.ctypes.data_as(ctypes.POINTER(ctypes.c_uint16)), b.size,
+                                  out.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
+    return out
 
 
 def heads(d, n_q, n_kv, d_h, wq_bits, wk_bits, v_in, iters, pairs, mode="factored",
@@ -194,4 +212,4 @@ def spectral_norms(wq_bits, wk_bits, v_in, iters, n_q, n_kv, d_h, mode="factored
 
 __all__ = ["calib", "form_interaction", "power_iteration_dense", "power_iteration_factored",
            "heads", "layer_implicit_gqa", "layer_form_expanded", "spectral_norms",
-           "max_threads", "LIB", "build"]
+           "max_threads", "LIB", "build", "set_weight_format", "decode_weights"]

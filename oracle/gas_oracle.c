@@ -7,10 +7,11 @@
  *
  * Notation (paper, Section 3.1 and Appendix E): for one attention head,
  *   W^Q_h, W^K_g in R^{d x d_h},  M = W^Q_h W^K_g^T in R^{d x d}  (Eq. 4, bilinear form).
- * Weights arrive in the nn.Linear layout: the d_h x d row-major bf16 block
+ * Weights arrive in the nn.Linear layout: the d_h x d row-major 16-bit block
  *   A[i][c] = W^Q_h[c][i]   (rows h*d_h .. h*d_h+d_h-1 of Wq),
- *   B[i][c] = W^K_g[c][i]   (rows g*d_h .. of Wk).
- * Every bf16 is widened exactly to double; all arithmetic is double.
+ *   B[i][c] = W^K_g[c][i]   (rows g*d_h .. of Wk),
+ * as bf16 (the default) or IEEE binary16 (oracle_set_weight_format(1)).  Every weight
+ * is widened exactly to double; all arithmetic is double.
  *
  * Power iteration, Algorithm 2 (Appendix E.1), one "iteration" =
  *   u' = M v;  sigma = ||u'||;  u = u'/sigma;  v' = M^T u;  v = v'/||v'||.
@@ -26,11 +27,37 @@
 #include <omp.h>
 #endif
 
+/* 0: bf16 (the top 16 bits of an IEEE binary32); 1: IEEE binary16. */
+static int g_weight_format = 0;
+
+void oracle_set_weight_format(int fmt) { g_weight_format = fmt; }
+
+/* binary16 by its definition: 1 sign bit, 5 exponent bits (bias 15), 10 fraction bits;
+ * exponent 0 holds the subnormals f * 2^-24, exponent 31 infinities and NaNs. */
+static double f16_bits_to_double(uint16_t bits)
+{
+    const int sign = (bits >> 15) & 1;
+    const int e = (bits >> 10) & 0x1F;
+    const int f = bits & 0x3FF;
+    double mag;
+    if (e == 0) mag = ldexp((double)f, -24);
+    else if (e == 31) mag = f ? NAN : INFINITY;
+    else mag = ldexp(1024.0 + f, e - 25);
+    return sign ? -mag : mag;
+}
+
 static double bf16_to_double(uint16_t bits)
 {
+    if (g_weight_format == 1) return f16_bits_to_double(bits);
     union { uint32_t u; float f; } x;
     x.u = ((uint32_t)bits) << 16;
     return (double)x.f;
+}
+
+/* Decode n weights of the current format (for tests of the decoder). */
+void oracle_decode_weights(const uint16_t *bits, long n, double *out)
+{
+    for (long i = 0; i < n; ++i) out[i] = bf16_to_double(bits[i]);
 }
 
 static double euclid_norm(const double *x, long n)

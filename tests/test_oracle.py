@@ -271,3 +271,37 @@ def test_bf16_widening_exact():
     bits = to_bf16_bits(x)
     t = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).double().numpy()
     np.testing.assert_array_equal(bits_to_f64(bits), t)
+
+
+def test_weight_decoders_exact_for_every_pattern():
+    """All 65536 bit patterns decode like numpy's binary16 and PyTorch's bfloat16."""
+    allb = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    try:
+        oracle.set_weight_format("f16")
+        got = oracle.decode_weights(allb)
+        want = allb.view(np.float16).astype(np.float64)
+        assert np.array_equal(np.isnan(got), np.isnan(want))
+        assert np.array_equal(got[~np.isnan(got)], want[~np.isnan(want)])
+    finally:
+        oracle.set_weight_format("bf16")
+    got = oracle.decode_weights(allb)
+    want = torch.from_numpy(allb.astype(np.int16)).view(torch.bfloat16).double().numpy()
+    assert np.array_equal(got[~np.isnan(got)], want[~np.isnan(want)])
+
+
+def test_f16_weights_match_svd_closed_form():
+    """Algorithm 2 on binary16 weights equals the SVD closed form of the exactly
+    decoded matrices (the bits are not reinterpreted as bf16)."""
+    rng = np.random.default_rng(16)
+    d, dh, k = 96, 8, 9
+    a = (rng.standard_normal((dh, d)) * 0.3).astype(np.float16)
+    b = (rng.standard_normal((dh, d)) * 0.3).astype(np.float16)
+    v0 = rng.standard_normal(d)
+    M = a.astype(np.float64).T @ b.astype(np.float64)
+    want, _, _, _, _ = sigma_k_closed_form(M, v0, k)
+    try:
+        oracle.set_weight_format("f16")
+        sig, _ = oracle.power_iteration_factored(a.view(np.uint16), b.view(np.uint16), v0, k)
+    finally:
+        oracle.set_weight_format("bf16")
+    assert sig == pytest.approx(want, rel=1e-10)
