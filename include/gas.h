@@ -158,8 +158,24 @@ double gas_alpha_min(double gamma, int d, int d_h, long long n_heads_total, int 
 gas_status gas_resolve_calibration(gas_handle h, double gamma, double delta_star,
                                    double *gamma_out, double *alpha_out);
 
+/* Element types (weights: gas_set_weight_dtype; logits: gas_fp8_quantize). */
+#define GAS_DTYPE_BF16 0
+#define GAS_DTYPE_F32  1
+#define GAS_DTYPE_F16  2
+
 /*
- * Weight layout (SURVEY row "layout generality"; the paper fixes none).  By default a
+ * Weight element type: GAS_DTYPE_BF16 (default) or GAS_DTYPE_F16 (IEEE binary16).  With
+ * binary16 weights the tensor-core operands (weights, and the hi + lo split start and
+ * write-back vectors) are binary16 too; sigma and v keep the same fp32 accumulation.
+ * The write-back's y / ||v'|| operand must lie inside binary16's range, which holds
+ * unless ||W^K_g||_2 is below about 2^-14.  Host only; applies to later calls.
+ * GAS_DTYPE_F32 -> GAS_ERR_UNSUPPORTED; anything else -> GAS_ERR_INVALID_ARG.
+ * gas_spectral_norms_static always reads bf16.
+ */
+gas_status gas_set_weight_dtype(gas_handle h, int dtype);
+
+/*
+ * Weight layout (the paper fixes none; it writes W^Q in R^{d x n_q d_h}).  By default a
  * layer's Wq[l] is the contiguous nn.Linear matrix [n_q * d_h, d].  Weights that are a
  * strided view of a larger allocation are described by two strides per matrix, in
  * elements:
@@ -167,14 +183,22 @@ gas_status gas_resolve_calibration(gas_handle h, double gamma, double delta_star
  * (likewise Wk[l] with ld_k, hs_k and key groups j).  This covers rows padded beyond d
  * (ld > d), and fused projections whose query and key blocks are interleaved per head,
  * e.g. [heads][3][d_h][d] gives ld = d, hs = 3 * d_h * d with Wk[l] = Wq[l] + d_h * d.
- *   layout  GAS_LAYOUT_ROWS (the only one implemented; others -> GAS_ERR_UNSUPPORTED)
- *   ld_q, ld_k  row strides, >= d; 0 = d
- *   hs_q, hs_k  head strides, >= d_h * row stride (heads do not overlap); 0 = d_h * ld
+ *   layout  GAS_LAYOUT_ROWS as above, or GAS_LAYOUT_COLS, the transposed (GPT-2
+ *           Conv1D) storage [d, n * d_h] with the output features contiguous:
+ *               element (row r = head * d_h + i, column c) at W[l][c * ld + r],
+ *           e.g. GPT-2's c_attn weight [d, 3d] gives Wq = W, Wk = W + d, ld = 3d.
+ *   ld_q, ld_k  ROWS: row strides, >= d; 0 = d.  COLS: column strides, >= n * d_h;
+ *               0 = n * d_h
+ *   hs_q, hs_k  ROWS: head strides, >= d_h * row stride (heads do not overlap);
+ *               0 = d_h * ld.  COLS: heads are contiguous, 0 or d_h only
  * All strides must be multiples of 8 elements (16-byte rows and heads, as TMA needs).
+ * GAS_LAYOUT_COLS is read by the tensor-core back ends (fused, gram); with it the
+ * streaming back end and gas_layer_refresh return GAS_ERR_UNSUPPORTED.
  * Host only; applies to every later call on the handle (gas_spectral_norms_static always
  * uses the contiguous layout).  Errors: GAS_ERR_INVALID_ARG with a message.
  */
 #define GAS_LAYOUT_ROWS 0
+#define GAS_LAYOUT_COLS 1
 gas_status gas_set_weight_layout(gas_handle h, int layout, long long ld_q, long long ld_k, long long hs_q,
                                  long long hs_k);
 

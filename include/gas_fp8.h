@@ -50,8 +50,7 @@ typedef struct gas_fp8_stats {
     unsigned long long count;     /* elements quantised */
 } gas_fp8_stats;
 
-#define GAS_DTYPE_BF16 0
-#define GAS_DTYPE_F32  1
+/* GAS_DTYPE_BF16 / GAS_DTYPE_F32 logits (defined in gas.h). */
 
 #define GAS_FP8_SATURATE 0x1      /* overflowing elements become +-448 (else NaN, 0x7F) */
 

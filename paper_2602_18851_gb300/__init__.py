@@ -105,6 +105,7 @@ def load(path: str = LIB_PATH):
     lib.gas_spectral_norms_static.argtypes = [c_int] * 5 + [vp, vp, c_int, vp, vp, vp, vp]
     lib.gas_layer_refresh.argtypes = [vp, vp, vp, c_int, vp, vp, vp, c_double, c_double, c_double, vp, vp]
     lib.gas_set_weight_layout.argtypes = [vp, c_int, c_ll, c_ll, c_ll, c_ll]
+    lib.gas_set_weight_dtype.argtypes = [vp, c_int]
     lib.gas_fp8_create.argtypes = [c_int, c_int, c_int, ctypes.POINTER(vp)]
     lib.gas_fp8_destroy.argtypes = [vp]
     lib.gas_fp8_reset.argtypes = [vp, ctypes.c_float, vp]
@@ -137,20 +138,25 @@ def alpha_min(gamma: float, d: int, d_h: int, n_heads_total: int, seq_len: int =
                                 float(delta_star))
 
 
-def _ptr_array(tensors: Sequence[torch.Tensor], rows: int, d: int, name: str, layout=None):
+def _ptr_array(tensors: Sequence[torch.Tensor], rows: int, d: int, name: str, layout=None,
+               dtype=torch.bfloat16):
     """Device pointers of per-layer weight tensors.  Default layout: each tensor is the
     contiguous [rows, d] matrix.  With a strided layout (heads, d_h, ld, hs) each tensor
     starts at the matrix's first element and must cover its last one."""
     arr = (ctypes.c_void_p * len(tensors))()
     for i, t in enumerate(tensors):
-        if t.dtype != torch.bfloat16 or not t.is_cuda:
-            raise ValueError(f"{name}[{i}] must be a CUDA bfloat16 tensor")
+        if t.dtype != dtype or not t.is_cuda:
+            raise ValueError(f"{name}[{i}] must be a CUDA {dtype} tensor")
         if layout is None:
             if not t.is_contiguous() or tuple(t.shape) != (rows, d):
                 raise ValueError(f"{name}[{i}] must be contiguous with shape {(rows, d)}, got {tuple(t.shape)}")
         else:
-            heads, dh, ld, hs = layout
-            last = (heads - 1) * hs + (dh - 1) * ld + d - 1
+            if layout[0] == "cols":
+                _, nrows, ld = layout
+                last = (d - 1) * ld + nrows - 1
+            else:
+                heads, dh, ld, hs = layout
+                last = (heads - 1) * hs + (dh - 1) * ld + d - 1
             avail = t.untyped_storage().nbytes() // 2 - t.storage_offset()
             if last >= avail:
                 raise ValueError(f"{name}[{i}]: the strided matrix needs {last + 1} elements, "
@@ -205,11 +211,18 @@ class Handle:
         _check(load().gas_set_calibration(self._h, int(seq_len), float(eta_fp8), float(alpha_override)),
                self._h)
 
-    def set_weight_layout(self, ld_q: int = 0, ld_k: int = 0, head_stride_q: int = 0, head_stride_k: int = 0):
-        """Strided weights (include/gas.h, gas_set_weight_layout): element (row i of head
-        j, column c) at w[j * head_stride + i * ld + c]; 0 keeps the contiguous default."""
-        _check(load().gas_set_weight_layout(self._h, 0, int(ld_q), int(ld_k), int(head_stride_q),
+    def set_weight_layout(self, ld_q: int = 0, ld_k: int = 0, head_stride_q: int = 0, head_stride_k: int = 0,
+                          layout: str = "rows"):
+        """Strided weights (include/gas.h, gas_set_weight_layout).  "rows": element (row i
+        of head j, column c) at w[j * head_stride + i * ld + c]; "cols" (GPT-2 Conv1D):
+        element (row r, column c) at w[c * ld + r].  0 keeps a default."""
+        code = {"rows": 0, "cols": 1}[layout]
+        _check(load().gas_set_weight_layout(self._h, code, int(ld_q), int(ld_k), int(head_stride_q),
                                             int(head_stride_k)), self._h)
+        if layout == "cols":
+            self._lq = ("cols", self.n_q * self.d_h, ld_q or self.n_q * self.d_h)
+            self._lk = ("cols", self.n_kv * self.d_h, ld_k or self.n_kv * self.d_h)
+            return
         lq = ld_q or self.d
         lk = ld_k or self.d
         hq = head_stride_q or lq * self.d_h
@@ -218,10 +231,18 @@ class Handle:
         self._lq = None if default else (self.n_q, self.d_h, lq, hq)
         self._lk = None if default else (self.n_kv, self.d_h, lk, hk)
 
+    def set_weight_dtype(self, dtype):
+        """Weight element type: "bf16" (default) or "f16" (torch dtypes accepted)."""
+        code = {"bf16": GAS_DTYPE_BF16, torch.bfloat16: GAS_DTYPE_BF16, "f16": GAS_DTYPE_F16,
+                torch.float16: GAS_DTYPE_F16, "f32": GAS_DTYPE_F32, torch.float32: GAS_DTYPE_F32}[dtype]
+        _check(load().gas_set_weight_dtype(self._h, code), self._h)
+        self._wdtype = torch.float16 if code == GAS_DTYPE_F16 else torch.bfloat16
+
     def _weights(self, wq, wk):
         lq, lk = getattr(self, "_lq", None), getattr(self, "_lk", None)
-        return (_ptr_array(wq, self.n_q * self.d_h, self.d, "wq", lq),
-                _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk", lk))
+        dt = getattr(self, "_wdtype", torch.bfloat16)
+        return (_ptr_array(wq, self.n_q * self.d_h, self.d, "wq", lq, dt),
+                _ptr_array(wk, self.n_kv * self.d_h, self.d, "wk", lk, dt))
 
     def set_method(self, method):
         m = METHODS[method] if isinstance(method, str) else int(method)
@@ -339,6 +360,7 @@ class Handle:
 
 GAS_DTYPE_BF16 = 0
 GAS_DTYPE_F32 = 1
+GAS_DTYPE_F16 = 2
 GAS_FP8_SATURATE = 0x1
 GAS_FP8_MAX_SLACK = 16384
 

@@ -129,6 +129,21 @@ bool encode_weights(CUtensorMap* m, const void* base, uint64_t d, uint32_t dh, u
   return r == CUDA_SUCCESS;
 }
 
+// 2D bf16 map of a Conv1D weight matrix: element (row r, column c) at base + c * ld + r;
+// box 64 rows x 64 columns (the rows are the contiguous, swizzled dimension).
+bool encode_cols(CUtensorMap* m, const void* base, uint64_t rows, uint64_t d, uint64_t ld) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {rows, d};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {64, 64};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 float scale_constant(const gas_ctx* h, double alpha, double r_max) {
   return static_cast<float>(alpha * (static_cast<double>(h->s.d) / std::sqrt(static_cast<double>(h->s.dh))) /
                             (h->eta_fp8 * r_max));
@@ -153,8 +168,12 @@ gas_status ensure_maps(gas_ctx* h, const void* const* wq, const void* const* wk,
   if (same) return GAS_OK;
   for (int l = 0; l < L; ++l) {
     const Shape& sh = h->s;
-    if (!encode_weights(&h->hmaps[l], wq[l], sh.d, sh.dh, sh.nq, sh.ldq, sh.hsq) ||
-        !encode_weights(&h->hmaps[L + l], wk[l], sh.d, sh.dh, sh.nkv, sh.ldk, sh.hsk))
+    const bool ok =
+        sh.cols ? encode_cols(&h->hmaps[l], wq[l], static_cast<uint64_t>(sh.nq) * sh.dh, sh.d, sh.ldq) &&
+                      encode_cols(&h->hmaps[L + l], wk[l], static_cast<uint64_t>(sh.nkv) * sh.dh, sh.d, sh.ldk)
+                : encode_weights(&h->hmaps[l], wq[l], sh.d, sh.dh, sh.nq, sh.ldq, sh.hsq) &&
+                      encode_weights(&h->hmaps[L + l], wk[l], sh.d, sh.dh, sh.nkv, sh.ldk, sh.hsk);
+    if (!ok)
       return fail(h, GAS_ERR_CUDA, "cuTensorMapEncodeTiled failed for layer %d", l);
     h->map_q[l] = wq[l];
     h->map_k[l] = wk[l];
@@ -341,6 +360,8 @@ gas_status spectral_impl(gas_ctx* h, const void* const* wq, const void* const* w
   std::memset(&tab, 0, sizeof(tab));
   fill_table(h, tab, wq, wk);
   const int method = h->method == GAS_METHOD_AUTO ? GAS_METHOD_FUSED : h->method;
+  if (method == GAS_METHOD_STREAM && h->s.cols)
+    return fail(h, GAS_ERR_UNSUPPORTED, "the streaming back end reads the nn.Linear layout only (use fused or gram)");
   if (method == GAS_METHOD_STREAM) return run_stream(h, tab, iters, v_in, v_out, sigma, s_out, scale_c, st);
   return run_gram(h, wq, wk, tab, iters, v_in, v_out, sigma, s_out, scale_c, method == GAS_METHOD_FUSED, st);
 }
@@ -452,6 +473,8 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   s.nz = nz_t;
   s.ldq = s.ldk = d;
   s.hsq = s.hsk = static_cast<long long>(d_h) * d;
+  s.f16 = 0;
+  s.cols = 0;
 
   cudaError_t e = cudaGetDevice(&h->device);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
@@ -568,24 +591,49 @@ gas_status gas_set_method(gas_handle h, int method) {
 gas_status gas_set_weight_layout(gas_handle h, int layout, long long ld_q, long long ld_k, long long hs_q,
                                  long long hs_k) {
   if (!h) return GAS_ERR_INVALID_ARG;
-  if (layout != GAS_LAYOUT_ROWS)
-    return fail(h, GAS_ERR_UNSUPPORTED, "layout %d is not implemented (only GAS_LAYOUT_ROWS)", layout);
   const Shape& s = h->s;
-  const long long lq = ld_q ? ld_q : s.d, lk = ld_k ? ld_k : s.d;
-  const long long hq = hs_q ? hs_q : lq * s.dh, hk = hs_k ? hs_k : lk * s.dh;
-  if (lq < s.d || lk < s.d)
-    return fail(h, GAS_ERR_INVALID_ARG, "row strides must be >= d (%d), got %lld and %lld", s.d, lq, lk);
-  if (hq < lq * s.dh || hk < lk * s.dh)
-    return fail(h, GAS_ERR_INVALID_ARG, "head strides must be >= d_h * row stride (heads must not overlap)");
+  long long lq, lk, hq, hk;
+  if (layout == GAS_LAYOUT_ROWS) {
+    lq = ld_q ? ld_q : s.d;
+    lk = ld_k ? ld_k : s.d;
+    hq = hs_q ? hs_q : lq * s.dh;
+    hk = hs_k ? hs_k : lk * s.dh;
+    if (lq < s.d || lk < s.d)
+      return fail(h, GAS_ERR_INVALID_ARG, "row strides must be >= d (%d), got %lld and %lld", s.d, lq, lk);
+    if (hq < lq * s.dh || hk < lk * s.dh)
+      return fail(h, GAS_ERR_INVALID_ARG, "head strides must be >= d_h * row stride (heads must not overlap)");
+  } else if (layout == GAS_LAYOUT_COLS) {
+    const long long rq = static_cast<long long>(s.nq) * s.dh, rk = static_cast<long long>(s.nkv) * s.dh;
+    lq = ld_q ? ld_q : rq;
+    lk = ld_k ? ld_k : rk;
+    if (lq < rq || lk < rk)
+      return fail(h, GAS_ERR_INVALID_ARG, "Conv1D strides must be >= the matrix's row count (%lld, %lld)", rq, rk);
+    if ((hs_q && hs_q != s.dh) || (hs_k && hs_k != s.dh))
+      return fail(h, GAS_ERR_INVALID_ARG, "Conv1D heads are contiguous: head strides must be 0 or d_h");
+    hq = hk = s.dh;
+  } else {
+    return fail(h, GAS_ERR_UNSUPPORTED, "unknown weight layout %d", layout);
+  }
   if (lq % 8 || lk % 8 || hq % 8 || hk % 8)
     return fail(h, GAS_ERR_INVALID_ARG, "row and head strides must be multiples of 8 elements (16 bytes)");
   if ((lq >> 37) || (lk >> 37) || (hq >> 37) || (hk >> 37))
     return fail(h, GAS_ERR_INVALID_ARG, "strides too large");
+  h->s.cols = layout == GAS_LAYOUT_COLS ? 1 : 0;
   h->s.ldq = lq;
   h->s.ldk = lk;
   h->s.hsq = hq;
   h->s.hsk = hk;
   h->maps_valid = false;  // descriptors are rebuilt at the next call
+  return GAS_OK;
+}
+
+gas_status gas_set_weight_dtype(gas_handle h, int dtype) {
+  if (!h) return GAS_ERR_INVALID_ARG;
+  if (dtype == GAS_DTYPE_F32)
+    return fail(h, GAS_ERR_UNSUPPORTED, "fp32 weights are not implemented (bf16 or fp16 only)");
+  if (dtype != GAS_DTYPE_BF16 && dtype != GAS_DTYPE_F16)
+    return fail(h, GAS_ERR_INVALID_ARG, "unknown weight dtype %d", dtype);
+  h->s.f16 = dtype == GAS_DTYPE_F16 ? 1 : 0;
   return GAS_OK;
 }
 
@@ -633,6 +681,8 @@ gas_status gas_layer_refresh(gas_handle h, const void* const* wq, const void* co
   if (!v_in || !sigma) return fail(h, GAS_ERR_INVALID_ARG, "v_in and sigma must not be NULL");
   if (!aligned16(v_in) || (v_out && !aligned16(v_out)))
     return fail(h, GAS_ERR_INVALID_ARG, "v_in / v_out must be 16-byte aligned");
+  if (h->s.cols)
+    return fail(h, GAS_ERR_UNSUPPORTED, "the whole-layer path reads the nn.Linear layout only");
   if (static_cast<size_t>(h->s.d + 8) * 4 > 227 * 1024 ||
       static_cast<size_t>(h->s.nq * h->s.dh + 2048) * 4 > 227 * 1024)
     return fail(h, GAS_ERR_UNSUPPORTED, "whole-layer path keeps a d- or n_q*d_h-vector in shared memory");

@@ -3,6 +3,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -21,6 +22,24 @@ __device__ __forceinline__ void unpack8(const uint4& q, float (&f)[8]) {
   f[2] = bf16lo(q.y); f[3] = bf16hi(q.y);
   f[4] = bf16lo(q.z); f[5] = bf16hi(q.z);
   f[6] = bf16lo(q.w); f[7] = bf16hi(q.w);
+}
+
+// Eight binary16 values (one 16-byte load) widened exactly to fp32.
+__device__ __forceinline__ void unpack8_f16(const uint4& q, float (&f)[8]) {
+  const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 v = __half22float2(*reinterpret_cast<const __half2*>(&w[i]));
+    f[2 * i] = v.x;
+    f[2 * i + 1] = v.y;
+  }
+}
+
+// Eight weights of the handle's format (bf16, or binary16 when F16).
+template <bool F16>
+__device__ __forceinline__ void unpack8w(const uint4& q, float (&f)[8]) {
+  if (F16) unpack8_f16(q, f);
+  else unpack8(q, f);
 }
 
 // Round-to-nearest-even fp32 -> bf16 bits.
@@ -283,12 +302,30 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 }
 
 // Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both K-major.
+// x as a hi + lo pair of 16-bit operands of the weights' format (bf16, or binary16):
+// hi = RN(x), lo = RN(x - hi).
+__device__ __forceinline__ void split_hilo(float x, bool f16, uint32_t& hb, uint32_t& lb) {
+  if (f16) {
+    const __half h = __float2half_rn(x);
+    hb = __half_as_ushort(h);
+    lb = __half_as_ushort(__float2half_rn(x - __half2float(h)));
+  } else {
+    hb = f32_to_bf16_bits(x);
+    lb = f32_to_bf16_bits(x - __uint_as_float(hb << 16));
+  }
+}
+
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4)                                 // D format: f32
          | (1u << 7)                               // A format: bf16
          | (1u << 10)                              // B format: bf16
          | (static_cast<uint32_t>(N >> 3) << 17)   // N / 8
          | (static_cast<uint32_t>(M >> 4) << 24);  // M / 16
+}
+
+// kind::f16 descriptor for bf16 (f16 == false) or binary16 operands (A and B alike).
+__host__ __device__ constexpr uint32_t idesc_f32acc(int M, int N, bool f16) {
+  return f16 ? (idesc_bf16_f32(M, N) & ~((1u << 7) | (1u << 10))) : idesc_bf16_f32(M, N);
 }
 
 // As idesc_bf16_f32 with A MN-major ("transpose A").

@@ -48,7 +48,7 @@ struct GramCfg {
   static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
 };
 
-// ---- v / ||v|| as bf16 hi + lo rows ---------------------------------------------------
+// ---- v / ||v|| as hi + lo rows of the weights' 16-bit format -----------------------
 // Row layout of one key tile's operand (nz rows): group gi of the tile owns rows
 // gi*2G .. gi*2G+2G-1; head j of the group has its hi part at gi*2G + j and its lo
 // part at gi*2G + G + j.  Padding rows stay zero (cleared at handle creation).
@@ -81,11 +81,7 @@ __global__ void __launch_bounds__(256) prep_v_kernel(const __grid_constant__ Pre
     const float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
     uint32_t hb[8], lb[8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const float xn = xv[e] * inv;
-      hb[e] = f32_to_bf16_bits(xn);
-      lb[e] = f32_to_bf16_bits(xn - __uint_as_float(hb[e] << 16));
-    }
+    for (int e = 0; e < 8; ++e) split_hilo(xv[e] * inv, s.f16 != 0, hb[e], lb[e]);
     *reinterpret_cast<uint4*>(hi_row + c) =
         make_uint4(hb[0] | (hb[1] << 16), hb[2] | (hb[3] << 16), hb[4] | (hb[5] << 16), hb[6] | (hb[7] << 16));
     *reinterpret_cast<uint4*>(lo_row + c) =
@@ -395,7 +391,12 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           const uint32_t sx = smem_u32(smem + st * SB);
           const uint32_t fb = smem_u32(&full[st]);
           mbar_arrive_expect_tx(fb, tr.is_k ? SB : kTileBytes);
-          tma_load_3d(sx, map, fb, kc * 64, 0, row0 / DH, pol);  // 128/d_h heads of d_h rows
+          if (s.cols) {  // out-features contiguous: two 64-row halves of the tile, MN-major
+            tma_load_2d(sx, map, fb, row0, kc * 64, pol);
+            tma_load_2d(sx + kTileBytes / 2, map, fb, row0 + 64, kc * 64, pol);
+          } else {
+            tma_load_3d(sx, map, fb, kc * 64, 0, row0 / DH, pol);  // 128/d_h heads of d_h rows
+          }
           if (tr.is_k) tma_load_2d(sx + kTileBytes, a.map_v, fb, kc * 64, vrow0, pol);
           ++issued;
         }
@@ -408,8 +409,9 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   } else if (warp == 1) {
     // ---------------- MMA issuer (one thread) ----------------
     if (lane == 0) {
-      constexpr uint32_t idG = idesc_bf16_f32(128, 128);
-      constexpr uint32_t idZ = idesc_bf16_f32(128, NZ);
+      // Conv1D weights arrive MN-major (A and B of G = X X^T, A of Z = X V^T).
+      const uint32_t idG = idesc_f32acc(128, 128, s.f16 != 0) | (s.cols ? (1u << 15) | (1u << 16) : 0u);
+      const uint32_t idZ = idesc_f32acc(128, NZ, s.f16 != 0) | (s.cols ? (1u << 15) : 0u);
       uint32_t consumed = 0, tc = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
@@ -424,13 +426,15 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sx = smem_u32(smem + st * SB);
-          const uint64_t ad = desc_kmajor_sw128(sx);
+          // K-major: +32 B per K16 step; MN-major (two 64-row atoms 8 KB apart): +2048 B
+          const uint64_t ad = s.cols ? desc_mnmajor_sw128_2atoms(sx, kTileBytes / 2) : desc_kmajor_sw128(sx);
+          const uint64_t astep = s.cols ? 128u : 2u;
           const uint64_t vd = desc_kmajor_sw128(sx + kTileBytes);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             const uint32_t accum = (kc | k) != 0 ? 1u : 0u;
-            umma_bf16(dG, ad + 2u * k, ad + 2u * k, idG, accum);
-            if (tr.is_k) umma_bf16(dZ, ad + 2u * k, vd + 2u * k, idZ, accum);
+            umma_bf16(dG, ad + astep * k, ad + astep * k, idG, accum);
+            if (tr.is_k) umma_bf16(dZ, ad + astep * k, vd + 2u * k, idZ, accum);
           }
           umma_commit(smem_u32(&empty[st]));
           ++consumed;

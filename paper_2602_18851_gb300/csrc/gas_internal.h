@@ -35,6 +35,8 @@ struct Shape {
   long long ldk;  // elements between consecutive rows of one key group of Wk[l] (>= d)
   long long hsq;  // elements between the first rows of consecutive query heads (>= d_h * ldq)
   long long hsk;  // elements between the first rows of consecutive key groups (>= d_h * ldk)
+  int f16;        // weights (and the MMA operands) are binary16 instead of bf16
+  int cols;       // GPT-2 Conv1D layout: element (row r, column c) at w[c * ld + r]
 };
 
 // Element offset of row r (head r / d_h, row r % d_h inside it) of a weight matrix.

@@ -21,7 +21,7 @@ __device__ __forceinline__ uint4 load_stream16(const uint16_t* p) {
   return __ldcs(reinterpret_cast<const uint4*>(p));
 }
 
-template <int DH, int MODE>
+template <int DH, int MODE, bool F16>
 __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant__ LayerTable tab,
                                                           const __grid_constant__ StreamArgs a) {
   constexpr int R = DH / 8;  // rows held per thread (warp w owns rows w, w+8, ...)
@@ -79,7 +79,7 @@ __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant_
 #pragma unroll
       for (int rr = 0; rr < R; ++rr) {
         float f[8];
-        unpack8(w[rr], f);
+        unpack8w<F16>(w[rr], f);
         const float xr = xs[warp + 8 * rr];
 #pragma unroll
         for (int c = 0; c < 8; ++c) pp[c] = fmaf(f[c], xr, pp[c]);
@@ -116,7 +116,7 @@ __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant_
 #pragma unroll
       for (int rr = 0; rr < R; ++rr) {
         float f[8];
-        unpack8(w[rr], f);
+        unpack8w<F16>(w[rr], f);
         float acc = 0.0f;
 #pragma unroll
         for (int c = 0; c < 8; ++c) acc = fmaf(f[c], p[c], acc);
@@ -169,18 +169,23 @@ __global__ void __launch_bounds__(32) scales_kernel(const __grid_constant__ Scal
   if (threadIdx.x == 0) a.s[l] = a.scale_c * m;
 }
 
-template <int DH>
-cudaError_t launch_stream_dh(const LayerTable& tab, const StreamArgs& a, cudaStream_t st) {
+template <int DH, bool F16>
+cudaError_t launch_stream_dt(const LayerTable& tab, const StreamArgs& a, cudaStream_t st) {
   const dim3 block(256);
   const dim3 grid(a.s.nch, a.mode == kPassQ ? a.s.nq : a.s.nkv, a.s.L);
   switch (a.mode) {
-    case kPassQ: stream_pass_kernel<DH, kPassQ><<<grid, block, 0, st>>>(tab, a); break;
-    case kPassK: stream_pass_kernel<DH, kPassK><<<grid, block, 0, st>>>(tab, a); break;
-    case kPassK0: stream_pass_kernel<DH, kPassK0><<<grid, block, 0, st>>>(tab, a); break;
-    case kPassKOut: stream_pass_kernel<DH, kPassKOut><<<grid, block, 0, st>>>(tab, a); break;
+    case kPassQ: stream_pass_kernel<DH, kPassQ, F16><<<grid, block, 0, st>>>(tab, a); break;
+    case kPassK: stream_pass_kernel<DH, kPassK, F16><<<grid, block, 0, st>>>(tab, a); break;
+    case kPassK0: stream_pass_kernel<DH, kPassK0, F16><<<grid, block, 0, st>>>(tab, a); break;
+    case kPassKOut: stream_pass_kernel<DH, kPassKOut, F16><<<grid, block, 0, st>>>(tab, a); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
+}
+
+template <int DH>
+cudaError_t launch_stream_dh(const LayerTable& tab, const StreamArgs& a, cudaStream_t st) {
+  return a.s.f16 ? launch_stream_dt<DH, true>(tab, a, st) : launch_stream_dt<DH, false>(tab, a, st);
 }
 
 }  // namespace

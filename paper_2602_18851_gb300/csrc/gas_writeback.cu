@@ -127,8 +127,19 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           const uint32_t fb = smem_u32(&full[st]);
           const uint32_t dst = smem_u32(ring + st * kStage);
           mbar_arrive_expect_tx(fb, kStage);
-          tma_load_3d(dst, &a.maps_k[w.layer], fb, w.c0 + 128 * j, 0, w.tile * (128 / DH), pol);
-          tma_load_3d(dst + kBox, &a.maps_k[w.layer], fb, w.c0 + 128 * j + 64, 0, w.tile * (128 / DH), pol);
+          if (s.cols) {
+            // Conv1D: box b holds rows (K) 64b.. of the tile for the 128 columns (M),
+            // K-major, fetched as two 64-column halves of 64-row boxes
+#pragma unroll
+            for (int b = 0; b < 2; ++b)
+#pragma unroll
+              for (int hh = 0; hh < 2; ++hh)
+                tma_load_2d(dst + b * kBox + hh * (kBox / 2), &a.maps_k[w.layer], fb, w.tile * 128 + 64 * b,
+                            w.c0 + 128 * j + 64 * hh, pol);
+          } else {
+            tma_load_3d(dst, &a.maps_k[w.layer], fb, w.c0 + 128 * j, 0, w.tile * (128 / DH), pol);
+            tma_load_3d(dst + kBox, &a.maps_k[w.layer], fb, w.c0 + 128 * j + 64, 0, w.tile * (128 / DH), pol);
+          }
           ++issued;
         }
       }
@@ -138,7 +149,8 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32_amn(128, NZ);
+      // A (the weight tile) is MN-major in the nn.Linear layout, K-major in the Conv1D one
+      const uint32_t idesc = idesc_f32acc(128, NZ, a.s.f16 != 0) | (a.s.cols ? 0u : (1u << 15));
       uint32_t consumed = 0, cc = 0, it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x, ++it) {
@@ -156,7 +168,8 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           const uint32_t sx = smem_u32(ring + st * kStage);
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            const uint64_t ad = desc_mnmajor_sw128_2atoms(sx + kk * 2048u, kBox);
+            const uint64_t ad = a.s.cols ? desc_kmajor_sw128(sx + (kk >> 2) * kBox + (kk & 3) * 32u)
+                                         : desc_mnmajor_sw128_2atoms(sx + kk * 2048u, kBox);
             const uint64_t bd = desc_kmajor_sw128(ybase + (kk >> 2) * (YB / 2) + (kk & 3) * 32u);
             umma_bf16(tmem + slot * NZ, ad, bd, idesc, kk > 0 ? 1u : 0u);
           }
@@ -203,8 +216,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           uint32_t hb[8], lb[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
-            hb[e] = f32_to_bf16_bits(v[e]);
-            lb[e] = f32_to_bf16_bits(v[e] - __uint_as_float(hb[e] << 16));
+            split_hilo(v[e], a.s.f16 != 0, hb[e], lb[e]);
           }
           const int k = gi * DH + i0;                     // K index of the 8-element chunk
           const int region = k >> 6, chunk = (k & 63) >> 3;

@@ -125,11 +125,12 @@ def _draw_layer(wl: Workload, layer: int, device, seed: int):
     return wq, wk, meta
 
 
-def make_weights(wl: Workload, device="cpu", seed: int | None = None
+def make_weights(wl: Workload, device="cpu", seed: int | None = None, dtype=torch.bfloat16
                  ) -> Tuple[List[torch.Tensor], List[torch.Tensor], Dict[str, torch.Tensor]]:
-    """bf16 weights of every layer, one tensor per layer and matrix.
+    """16-bit weights of every layer (bf16 by default, or float16), one tensor per layer
+    and matrix, rounded to nearest from the same unrounded draw.
 
-    Returns (wq, wk, meta): wq[l] is ``[n_q*d_h, d]`` bf16, wk[l] is ``[n_kv*d_h, d]``.
+    Returns (wq, wk, meta): wq[l] is ``[n_q*d_h, d]``, wk[l] is ``[n_kv*d_h, d]``.
     For the ``planted`` recipe ``meta`` holds per-head ``sigma_planted``, ``norm_q``,
     ``norm_k`` ([layers, ...] float64) and the Frobenius norms of the bf16 rounding
     residuals ``err_q``/``err_k`` used for the Weyl perturbation bound.
@@ -138,7 +139,7 @@ def make_weights(wl: Workload, device="cpu", seed: int | None = None
     wq, wk, metas = [], [], []
     for layer in range(wl.layers):
         q, k, meta = _draw_layer(wl, layer, device, seed)
-        qb, kb = q.to(torch.bfloat16), k.to(torch.bfloat16)
+        qb, kb = q.to(dtype), k.to(dtype)
         if wl.recipe == "planted":
             eq = (qb.double() - q.double()).view(wl.n_q, wl.d_h, wl.d).norm(dim=(1, 2))
             ek = (kb.double() - k.double()).view(wl.n_kv, wl.d_h, wl.d).norm(dim=(1, 2))

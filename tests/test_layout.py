@@ -118,7 +118,7 @@ def test_layout_argument_errors():
     wl = get_workload("tiny-gqa128")
     with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
         lib = gas.load()
-        assert lib.gas_set_weight_layout(h._h, 1, 0, 0, 0, 0) == gas.GAS_ERR_UNSUPPORTED
+        assert lib.gas_set_weight_layout(h._h, 5, 0, 0, 0, 0) == gas.GAS_ERR_UNSUPPORTED
         assert lib.gas_set_weight_layout(h._h, 0, wl.d - 8, 0, 0, 0) == gas.GAS_ERR_INVALID_ARG
         assert lib.gas_set_weight_layout(h._h, 0, wl.d + 4, 0, 0, 0) == gas.GAS_ERR_INVALID_ARG
         assert lib.gas_set_weight_layout(h._h, 0, 0, 0, wl.d * wl.d_h - 8, 0) == gas.GAS_ERR_INVALID_ARG
@@ -128,3 +128,54 @@ def test_layout_argument_errors():
         h.set_weight_layout(ld_q=wl.d + 64)
         with pytest.raises(ValueError):
             h.refresh(wq, wk, 2, v_in)  # the contiguous tensors do not cover the strided extent
+
+
+def _conv1d(wq, wk, pad_cols):
+    """GPT-2 Conv1D storage: one [d, n_q*d_h + n_kv*d_h + pad] tensor per layer holding
+    W^Q (columns 0..), W^K (next columns) and NaN padding; output features contiguous."""
+    qs, ks, ld = [], [], None
+    for q, k in zip(wq, wk):
+        rq, d = q.shape
+        rk = k.shape[0]
+        ld = rq + rk + pad_cols
+        buf = torch.full((d, ld), float("nan"), dtype=q.dtype, device=q.device)
+        buf[:, :rq] = q.t()
+        buf[:, rq:rq + rk] = k.t()
+        flat = buf.view(-1)
+        qs.append(flat)
+        ks.append(flat[rq:])
+    return qs, ks, ld
+
+
+@pytest.mark.parametrize("name", ["gpt2-small", "tiny-gqa128", "tiny-gqa", "ragged", "tiny-g32"])
+@pytest.mark.parametrize("method", ["fused", "gram"])
+def test_conv1d_layout_matches_oracle(name, method):
+    """Transposed (Conv1D) weights run through MN-major tensor-core operands; sigma, the
+    scales and v_out agree with the contiguous run and with the oracle."""
+    wl = get_workload(name)
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    ref = _run(wl, wq, wk, v_in, method)
+    cq, ck, ld = _conv1d(wq, wk, pad_cols=8 * ((wl.n_kv * wl.d_h) // 8))
+    got = _run(wl, cq, ck, v_in, method, layout=dict(ld_q=ld, ld_k=ld, layout="cols"))
+    np.testing.assert_allclose(got[0].numpy(), ref[0].numpy(), rtol=1e-5)
+    np.testing.assert_allclose(got[1].numpy(), ref[1].numpy(), rtol=1e-5)
+    assert float((got[2] - ref[2]).norm(dim=-1).max()) < 1e-4
+    sig_ref, _ = oracle_for(wl, wq, wk, v_in)
+    assert_sigma_close(got[0].double().numpy().ravel(), sig_ref.ravel(), rtol=SIGMA_RTOL)
+
+
+def test_conv1d_layout_rejected_by_streaming_and_whole_layer_paths():
+    wl = get_workload("tiny-gqa128")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    cq, ck, ld = _conv1d(wq, wk, 0)
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        h.set_weight_layout(ld_q=ld, ld_k=ld, layout="cols")
+        h.set_method("stream")
+        with pytest.raises(gas.GasError) as e:
+            h.refresh(cq, ck, 2, v_in)
+        assert e.value.status == gas.GAS_ERR_UNSUPPORTED
+        with pytest.raises(gas.GasError):
+            h.layer_refresh(cq, ck, 2, v_in[:, 0, :].contiguous())
+        lib = gas.load()
+        assert lib.gas_set_weight_layout(h._h, 1, wl.n_q * wl.d_h - 8, 0, 0, 0) == gas.GAS_ERR_INVALID_ARG
+        assert lib.gas_set_weight_layout(h._h, 1, 0, 0, 2 * wl.d_h, 0) == gas.GAS_ERR_INVALID_ARG
