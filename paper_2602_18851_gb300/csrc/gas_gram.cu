@@ -327,7 +327,9 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
   }
 }
 
-template <int NZ, int DH, bool FUSED>
+// GENERIC: binary16 weights or the Conv1D layout, chosen at run time; the default
+// instantiation (bf16, nn.Linear rows) has both folded away.
+template <int NZ, int DH, bool FUSED, bool GENERIC>
 __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(const __grid_constant__ GramArgs a) {
   constexpr int NE = 32 * GramWarps<FUSED>::kEpiWarps;  // epilogue threads
   using Cfg = GramCfg<NZ>;
@@ -350,6 +352,8 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   volatile int no_abort_flag = 0;
 
   const Shape& s = a.s;
+  const bool cols = GENERIC && s.cols != 0;
+  const bool f16 = GENERIC && s.f16 != 0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -391,7 +395,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           const uint32_t sx = smem_u32(smem + st * SB);
           const uint32_t fb = smem_u32(&full[st]);
           mbar_arrive_expect_tx(fb, tr.is_k ? SB : kTileBytes);
-          if (s.cols) {  // out-features contiguous: two 64-row halves of the tile, MN-major
+          if (cols) {  // out-features contiguous: two 64-row halves of the tile, MN-major
             tma_load_2d(sx, map, fb, row0, kc * 64, pol);
             tma_load_2d(sx + kTileBytes / 2, map, fb, row0 + 64, kc * 64, pol);
           } else {
@@ -410,8 +414,8 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     // ---------------- MMA issuer (one thread) ----------------
     if (lane == 0) {
       // Conv1D weights arrive MN-major (A and B of G = X X^T, A of Z = X V^T).
-      const uint32_t idG = idesc_f32acc(128, 128, s.f16 != 0) | (s.cols ? (1u << 15) | (1u << 16) : 0u);
-      const uint32_t idZ = idesc_f32acc(128, NZ, s.f16 != 0) | (s.cols ? (1u << 15) : 0u);
+      const uint32_t idG = idesc_f32acc(128, 128, f16) | (cols ? (1u << 15) | (1u << 16) : 0u);
+      const uint32_t idZ = idesc_f32acc(128, NZ, f16) | (cols ? (1u << 15) : 0u);
       uint32_t consumed = 0, tc = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
@@ -427,8 +431,8 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           tc_fence_after();
           const uint32_t sx = smem_u32(smem + st * SB);
           // K-major: +32 B per K16 step; MN-major (two 64-row atoms 8 KB apart): +2048 B
-          const uint64_t ad = s.cols ? desc_mnmajor_sw128_2atoms(sx, kTileBytes / 2) : desc_kmajor_sw128(sx);
-          const uint64_t astep = s.cols ? 128u : 2u;
+          const uint64_t ad = cols ? desc_mnmajor_sw128_2atoms(sx, kTileBytes / 2) : desc_kmajor_sw128(sx);
+          const uint64_t astep = cols ? 128u : 2u;
           const uint64_t vd = desc_kmajor_sw128(sx + kTileBytes);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
@@ -616,10 +620,10 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
   }
 }
 
-template <int NZ, int DH, bool FUSED>
+template <int NZ, int DH, bool FUSED, bool GENERIC>
 cudaError_t launch_gram_cfg(const GramArgs& a, int num_sms, cudaStream_t st) {
   using Cfg = GramCfg<NZ>;
-  auto kern = gram_kernel<NZ, DH, FUSED>;
+  auto kern = gram_kernel<NZ, DH, FUSED, GENERIC>;
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -642,12 +646,18 @@ cudaError_t launch_gram_cfg(const GramArgs& a, int num_sms, cudaStream_t st) {
   return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
+template <int NZ, int DH, bool FUSED>
+cudaError_t launch_gram_variant(const GramArgs& a, int num_sms, cudaStream_t st) {
+  return (a.s.cols || a.s.f16) ? launch_gram_cfg<NZ, DH, FUSED, true>(a, num_sms, st)
+                               : launch_gram_cfg<NZ, DH, FUSED, false>(a, num_sms, st);
+}
+
 template <int NZ>
 cudaError_t launch_gram_nz(const GramArgs& a, int num_sms, bool fused, cudaStream_t st) {
   if (a.s.dh == 128)
-    return fused ? launch_gram_cfg<NZ, 128, true>(a, num_sms, st) : launch_gram_cfg<NZ, 128, false>(a, num_sms, st);
+    return fused ? launch_gram_variant<NZ, 128, true>(a, num_sms, st) : launch_gram_variant<NZ, 128, false>(a, num_sms, st);
   if (a.s.dh == 64)
-    return fused ? launch_gram_cfg<NZ, 64, true>(a, num_sms, st) : launch_gram_cfg<NZ, 64, false>(a, num_sms, st);
+    return fused ? launch_gram_variant<NZ, 64, true>(a, num_sms, st) : launch_gram_variant<NZ, 64, false>(a, num_sms, st);
   return cudaErrorInvalidValue;
 }
 

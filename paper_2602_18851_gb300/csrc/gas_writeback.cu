@@ -56,7 +56,9 @@ __device__ __forceinline__ WbItem decode_item(const Shape& s, int t) {
   return w;
 }
 
-template <int DH, int NZ>
+// GENERIC: binary16 weights or the Conv1D layout, chosen at run time (folded away in the
+// default bf16 nn.Linear instantiation).
+template <int DH, int NZ, bool GENERIC>
 __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_constant__ WbArgs a) {
   using Cfg = WbCfg<NZ>;
   constexpr int S = Cfg::kStages;
@@ -81,6 +83,8 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
   volatile int no_abort_flag = 0;
 
   const Shape& s = a.s;
+  const bool cols = GENERIC && s.cols != 0;
+  const bool f16 = GENERIC && s.f16 != 0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -127,7 +131,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           const uint32_t fb = smem_u32(&full[st]);
           const uint32_t dst = smem_u32(ring + st * kStage);
           mbar_arrive_expect_tx(fb, kStage);
-          if (s.cols) {
+          if (cols) {
             // Conv1D: box b holds rows (K) 64b.. of the tile for the 128 columns (M),
             // K-major, fetched as two 64-column halves of 64-row boxes
 #pragma unroll
@@ -150,7 +154,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
   } else if (warp == 1) {
     if (lane == 0) {
       // A (the weight tile) is MN-major in the nn.Linear layout, K-major in the Conv1D one
-      const uint32_t idesc = idesc_f32acc(128, NZ, a.s.f16 != 0) | (a.s.cols ? 0u : (1u << 15));
+      const uint32_t idesc = idesc_f32acc(128, NZ, f16) | (cols ? 0u : (1u << 15));
       uint32_t consumed = 0, cc = 0, it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x, ++it) {
@@ -168,7 +172,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           const uint32_t sx = smem_u32(ring + st * kStage);
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            const uint64_t ad = a.s.cols ? desc_kmajor_sw128(sx + (kk >> 2) * kBox + (kk & 3) * 32u)
+            const uint64_t ad = cols ? desc_kmajor_sw128(sx + (kk >> 2) * kBox + (kk & 3) * 32u)
                                          : desc_mnmajor_sw128_2atoms(sx + kk * 2048u, kBox);
             const uint64_t bd = desc_kmajor_sw128(ybase + (kk >> 2) * (YB / 2) + (kk & 3) * 32u);
             umma_bf16(tmem + slot * NZ, ad, bd, idesc, kk > 0 ? 1u : 0u);
@@ -216,7 +220,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           uint32_t hb[8], lb[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
-            split_hilo(v[e], a.s.f16 != 0, hb[e], lb[e]);
+            split_hilo(v[e], f16, hb[e], lb[e]);
           }
           const int k = gi * DH + i0;                     // K index of the 8-element chunk
           const int region = k >> 6, chunk = (k & 63) >> 3;
@@ -284,12 +288,12 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
   }
 }
 
-template <int DH, int NZ>
-cudaError_t launch_wb_cfg(const WbArgs& a, int num_sms, cudaStream_t st) {
+template <int DH, int NZ, bool GENERIC>
+cudaError_t launch_wb_gen(const WbArgs& a, int num_sms, cudaStream_t st) {
   using Cfg = WbCfg<NZ>;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(writeback_kernel<DH, NZ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(writeback_kernel<DH, NZ, GENERIC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(Cfg::kSmem));
     if (e != cudaSuccess) return e;
     configured = true;
@@ -297,8 +301,13 @@ cudaError_t launch_wb_cfg(const WbArgs& a, int num_sms, cudaStream_t st) {
   const int ncb = (a.s.d + kWbCols - 1) / kWbCols;
   const int T = a.s.L * a.s.tiles_k * ncb;
   const int grid = T < num_sms ? T : num_sms;
-  writeback_kernel<DH, NZ><<<grid, kWbThreads, Cfg::kSmem, st>>>(a);
+  writeback_kernel<DH, NZ, GENERIC><<<grid, kWbThreads, Cfg::kSmem, st>>>(a);
   return cudaGetLastError();
+}
+
+template <int DH, int NZ>
+cudaError_t launch_wb_cfg(const WbArgs& a, int num_sms, cudaStream_t st) {
+  return (a.s.cols || a.s.f16) ? launch_wb_gen<DH, NZ, true>(a, num_sms, st) : launch_wb_gen<DH, NZ, false>(a, num_sms, st);
 }
 
 template <int DH>
