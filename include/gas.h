@@ -24,6 +24,12 @@
  *  - Calls that take a stream are asynchronous and stream-ordered; the host checks
  *    arguments synchronously and enqueues nothing on error.  `stream` is a
  *    cudaStream_t (NULL = legacy default stream).
+ *  - CUDA graphs: the first call with a new set of weight pointers (or after
+ *    gas_set_weight_layout) builds their TMA descriptors and synchronises the stream
+ *    once to upload them; every later call with the same pointers is pure stream work
+ *    and can be captured (cudaStreamBeginCapture) and replayed.  Replays read the
+ *    weights and v_in afresh; the fused kernel's key-tile flags take a new value on
+ *    every replay (advanced on the device), so replays never see stale Gram blocks.
  *  - No exceptions cross this boundary.  A handle is not thread-safe; concurrent
  *    calls on one handle (or overlapping launches of one handle on two streams)
  *    race on its workspace.

@@ -51,7 +51,7 @@ struct gas_ctx {
   float* lu = nullptr;           //                   u'   [L][d]
   float* ly = nullptr;           //                   y    [L][n_q*d_h]
   float* lv = nullptr;           //                   v'   [L][d]
-  unsigned epoch = 0;            // last flag value used
+  unsigned* epoch = nullptr;     // device word: flag value of the fused Gram launches
 
   // host copies of the encoded descriptors and the pointers they were built for
   std::vector<CUtensorMap> hmaps;
@@ -287,6 +287,7 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
   p.v_in = v_in;
   p.vhl = h->vhl;
   p.s_zero = s_out;
+  p.epoch = h->epoch;
   cudaError_t e = launch(h, "prep_v", st, [&] { return gas::launch_prep_v(p, st); });
   ++launches;
   if (e == cudaSuccess) {
@@ -300,7 +301,6 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
     g.z0 = h->z0;
     g.status = h->status;
     if (fused) {
-      h->epoch = h->epoch == 0xFFFFFFFFu ? 1u : h->epoch + 1u;
       g.flags = h->flags;
       g.epoch = h->epoch;
       g.iters = iters;
@@ -499,7 +499,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
     off = align_up(off + bytes, 256);
     return o;
   };
-  const size_t o_status = take(256);
+  const size_t o_status = take(256);  // status word, then the epoch word at +128
   const size_t o_zp = take(L * NQ * NCH * DH * 4);
   const size_t o_n2p = take(L * NQ * NCH * 4);
   const size_t o_tp = take(L * NQ * NCH * DH * 4);
@@ -524,6 +524,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   e = cudaMemset(h->ws, 0, h->ws_bytes);
   char* b = static_cast<char*>(h->ws);
   h->status = reinterpret_cast<unsigned*>(b + o_status);
+  h->epoch = reinterpret_cast<unsigned*>(b + o_status + 128);
   h->zp = reinterpret_cast<float*>(b + o_zp);
   h->n2p = reinterpret_cast<float*>(b + o_n2p);
   h->tp = reinterpret_cast<float*>(b + o_tp);

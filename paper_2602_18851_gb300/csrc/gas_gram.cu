@@ -88,6 +88,10 @@ __global__ void __launch_bounds__(256) prep_v_kernel(const __grid_constant__ Pre
         make_uint4(lb[0] | (lb[1] << 16), lb[2] | (lb[3] << 16), lb[4] | (lb[5] << 16), lb[6] | (lb[7] << 16));
   }
   if (a.s_zero != nullptr && h == 0 && threadIdx.x == 0) a.s_zero[l] = 0.0f;
+  if (hidx == 0 && threadIdx.x == 0 && a.epoch != nullptr) {
+    const unsigned e = *a.epoch + 1u;
+    *a.epoch = e == 0u ? 1u : e;
+  }
 }
 
 // ---- tcgen05 Gram kernel -------------------------------------------------------------
@@ -177,7 +181,7 @@ __device__ __forceinline__ float halfwarp_transpose_reduce8(float (&v)[8], int l
 template <int DH>
 __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int idx, uint32_t tacc, int q,
                                               int half, int ew, int lane, EpiSmem* ep, volatile int* abort,
-                                              uint32_t acce_bar) {
+                                              uint32_t acce_bar, unsigned epoch) {
   constexpr int HPT = 128 / DH;   // heads per 128-row tile
   constexpr int NTH = 256 / HPT;  // threads per head
   constexpr int NWH = NTH / 32;   // warps per head
@@ -238,7 +242,7 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
   const int g = head / s.G;
   const int tk = (g * DH) / 128, og = (g * DH) % 128;
   const unsigned* flag = a.flags + layer * s.tiles_k + tk;
-  if (th == 0) ep->ok[hs] = wait_flag(flag, a.epoch, abort, a.status) ? 1 : 0;
+  if (th == 0) ep->ok[hs] = wait_flag(flag, epoch, abort, a.status) ? 1 : 0;
   named_bar_sync(bar, NTH);
   if (!ep->ok[hs]) return;
   (void)ld_acquire_u32(flag);
@@ -459,6 +463,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     constexpr int CW = 128 * 128 / NE;  // accumulator columns per thread when storing G
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const int gpt = 128 / s.dh;
+    const unsigned epoch = FUSED ? __ldcg(a.epoch) : 0u;
     uint32_t tc = 0;
     for (int t = blockIdx.x; t < T; t += gridDim.x) {
       const TileRef tr = decode_tile(s, t);
@@ -471,7 +476,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       tc_fence_after();
       if (FUSED && !tr.is_k) {  // (hands the accumulator back itself, right after reading G_Q)
         fused_iterate<DH>(a, tr.layer, tr.idx, tmem + lane_off + acc * 128u, q, half, warp - 2, lane, ep,
-                          abort, smem_u32(&acce[acc]));
+                          abort, smem_u32(&acce[acc]), epoch);
         ++tc;
         continue;
       }
@@ -509,7 +514,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       if (FUSED && tr.is_k) {  // publish G_K and z0 of this key tile to the query tiles' epilogues
         __threadfence();
         named_bar_sync(3, NE);
-        if (row == 0 && half == 0) st_release_u32(a.flags + tr.layer * s.tiles_k + tr.idx, a.epoch);
+        if (row == 0 && half == 0) st_release_u32(a.flags + tr.layer * s.tiles_k + tr.idx, epoch);
       }
       tc_fence_before();
       mbar_arrive(smem_u32(&acce[acc]));

@@ -86,6 +86,7 @@ struct PrepArgs {
   const float* v_in;   // [L][nq][d]
   uint16_t* vhl;       // [L][tiles_k][nz][d] bf16 hi/lo rows of v / ||v||
   float* s_zero;       // [L] or null
+  unsigned* epoch;     // flag value of the next fused Gram launch (advanced here)
 };
 
 struct GramArgs {
@@ -99,7 +100,8 @@ struct GramArgs {
   unsigned* status;
   // fused variant: k iterations in the epilogue, straight from tensor memory
   unsigned* flags;            // [L][tiles_k] key-tile publication flags (== epoch when ready)
-  unsigned epoch;             // this launch's flag value (never 0)
+  const unsigned* epoch;      // this launch's flag value (never 0), advanced on the device by
+                              // prep_v_kernel, so that a replayed CUDA graph gets a new one
   int iters;
   float* ybuf;                // [L][nq][dh]
   float* sigma;               // [L][nq]
