@@ -9,6 +9,8 @@ are resident in HBM and larger than L2, so no L2 flush is needed between steps.
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                     [--workload NAME] [--method auto|gram|stream] [--path refresh|e4m3]
 
+--path layer times the whole-layer sigma (gas_layer_refresh) instead; --dtype f16 and
+--layout padded|cols time the same refresh on binary16 or strided / Conv1D weights.
 --path e4m3 measures the scale's consumer instead: one gas_fp8_quantize call (Algorithm
 1, Stage 3) on one Llama-2-70B layer's logits at batch 2 x seq 1024 (2 x 64 x 1024 x
 1024 bf16, 268 MB > L2), cast to E4M3 with its overflow statistics.
@@ -36,6 +38,7 @@ if ROOT not in sys.path:
 from synth import get_workload, make_start_vectors, make_weights  # noqa: E402
 
 METRIC = "full-model sigma+scale refresh ms (Llama-2-70B GQA shape); % of HBM roofline"
+METRIC_LAYER = "whole-layer sigma+scale refresh ms (Algorithms 2-3 as printed); % of HBM roofline of its passes"
 METRIC_E4M3 = "E4M3 cast of one Llama-2-70B layer's attention logits (2x64x1024x1024 bf16) ms; % of HBM roofline"
 
 
@@ -52,7 +55,12 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU-baseline sample budget")
-    p.add_argument("--path", default="refresh", choices=["refresh", "e4m3"])
+    p.add_argument("--path", default="refresh", choices=["refresh", "e4m3", "layer"],
+                   help="refresh: per-head sigma + scales (default); layer: whole-layer sigma "
+                        "(Algorithms 2-3 as printed); e4m3: the scales' consumer")
+    p.add_argument("--dtype", default="bf16", choices=["bf16", "f16"], help="weight element type")
+    p.add_argument("--layout", default="rows", choices=["rows", "padded", "cols"],
+                   help="weight storage: nn.Linear rows, rows padded by 64 elements, GPT-2 Conv1D")
     return p.parse_args()
 
 
@@ -221,6 +229,31 @@ def oracle_sample_ms(wl, iters, budget_s, wq=None, wk=None, v_in=None):
             "sample": f"{heads} heads ({layers_done} whole layers) of {wl.name}, {iters} iterations, "
                       f"float64 factored power iteration incl. v write-back, {spent:.1f} s; "
                       f"extrapolated linearly to all {wl.heads} heads"}
+
+
+def arrange_weights(h, wl, wq, wk, layout):
+    """Store the weights as `layout` asks and tell the handle: nn.Linear rows (as drawn),
+    rows padded by 64 elements, or the GPT-2 Conv1D storage [d, n_q*d_h + n_kv*d_h]."""
+    if layout == "rows":
+        return wq, wk
+    qs, ks = [], []
+    if layout == "padded":
+        for q, k in zip(wq, wk):
+            qs.append(torch.nn.functional.pad(q, (0, 64)))
+            ks.append(torch.nn.functional.pad(k, (0, 64)))
+        h.set_weight_layout(ld_q=wl.d + 64, ld_k=wl.d + 64)
+        return qs, ks
+    rq, rk = wl.n_q * wl.d_h, wl.n_kv * wl.d_h
+    for i in range(len(wq)):
+        buf = torch.empty((wl.d, rq + rk), dtype=wq[i].dtype, device=wq[i].device)
+        buf[:, :rq] = wq[i].t()
+        buf[:, rq:] = wk[i].t()
+        flat = buf.view(-1)
+        qs.append(flat)
+        ks.append(flat[rq:])
+        wq[i] = wk[i] = None
+    h.set_weight_layout(ld_q=rq + rk, ld_k=rq + rk, layout="cols")
+    return qs, ks
 
 
 def e4m3_logits_shape():
@@ -418,17 +451,28 @@ def main():
     if args.layers:
         wl = wl.scaled(layers=args.layers)
     iters = args.iters or wl.iters
-    wq, wk, _ = make_weights(wl, device=dev)
-    v_in = make_start_vectors(wl, device=dev)
-    v_out = torch.empty_like(v_in)
-    sigma = torch.empty(wl.layers, wl.n_q, device=dev)
-    s = torch.empty(wl.layers, device=dev)
+    wdt = torch.float16 if args.dtype == "f16" else torch.bfloat16
+    wq, wk, _ = make_weights(wl, device=dev, dtype=wdt)
     h = gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h)
     h.set_method(args.method)
+    if args.dtype == "f16":
+        h.set_weight_dtype("f16")
+    wq, wk = arrange_weights(h, wl, wq, wk, args.layout)
+    v_in = make_start_vectors(wl, device=dev)
+    if args.path == "layer":
+        v_in = v_in[:, 0, :].contiguous()
+        sigma = torch.empty(wl.layers, device=dev)
+    else:
+        sigma = torch.empty(wl.layers, wl.n_q, device=dev)
+    v_out = torch.empty_like(v_in)
+    s = torch.empty(wl.layers, device=dev)
     stream = torch.cuda.current_stream(dev)
 
     def step():
-        h.refresh(wq, wk, iters, v_in, v_out=v_out, sigma=sigma, s=s)
+        if args.path == "layer":
+            h.layer_refresh(wq, wk, iters, v_in, v_out=v_out, sigma=sigma, s=s)
+        else:
+            h.refresh(wq, wk, iters, v_in, v_out=v_out, sigma=sigma, s=s)
 
     for _ in range(max(3, args.warmup)):
         step()
@@ -471,7 +515,17 @@ def main():
     v_b = 4 * wl.layers * wl.n_q * wl.d
     algo_step = weight_b + 2 * v_b
     method = "fused" if "gram_fused" in names else ("gram" if "gram" in names else "stream")
-    if method in ("fused", "gram"):
+    if args.path == "layer":
+        # Algorithms 2-3 as printed: four weight passes per iteration (k_rowdot, q_coldot,
+        # q_rowdot, k_coldot); the least such a k-step run moves is those passes
+        method = "layer"
+        v_b = 4 * wl.layers * wl.d
+        algo_step = iters * 2 * weight_b + 2 * v_b
+        dom = "layer_rowdot_q"
+        n_l = launches.get(dom, 1)
+        dom_bytes = 2 * wl.layers * wl.n_q * wl.d_h * wl.d  # one W^Q pass per launch
+        dom_ms = kern_ms[dom] / n_l
+    elif method in ("fused", "gram"):
         dom = "gram_fused" if method == "fused" else "gram"
         dom_bytes = weight_b + v_b     # every W^Q_h and W^K_g once + the start vectors
         dom_ms = kern_ms[dom]
@@ -486,7 +540,7 @@ def main():
     # end to end through the public API with host buffers: H2D weights + v_in every step,
     # refresh, D2H of sigma, scales and v_out
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and args.path == "refresh" and args.layout == "rows":
         hq = [w.cpu().pin_memory() for w in wq]
         hk = [w.cpu().pin_memory() for w in wk]
         hv = v_in.cpu().pin_memory()
@@ -521,17 +575,20 @@ def main():
         del hq, hk, hv
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if (rank == 0 and world == 1 and not args.no_cpu_baseline and args.path == "refresh"
+            and args.layout == "rows" and args.dtype == "bf16"):
         cpu = oracle_sample_ms(wl, iters, args.cpu_seconds, wq=wq, wk=wk, v_in=v_in)
 
     if rank == 0:
         out = {
-            "metric": METRIC, "value": ms, "unit": "ms", "n_gpus": world, "steps": K,
+            "metric": METRIC if args.path == "refresh" else METRIC_LAYER, "value": ms, "unit": "ms",
+            "n_gpus": world, "steps": K,
             "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": False,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16 weights, f32 accumulate",
+            "scaling": "weak", "vs_baseline": None, "dtype": f"{args.dtype} weights, f32 accumulate",
             "data": "synthetic",
             "config": {"workload": wl.name, "layers": wl.layers, "d": wl.d, "n_q": wl.n_q,
                        "n_kv": wl.n_kv, "d_h": wl.d_h, "iters": iters, "method": method,
+                       "path": args.path, "weight_layout": args.layout,
                        "parallelism": "replicas" if world > 1 else "single-gpu",
                        "l2": "inputs 12.4 GB > 129 MB L2, no flush needed"},
             "hbm_roofline_pct": 100.0 * step_gbs / peak,
