@@ -595,7 +595,9 @@ def main():
             "step_achieved_gbs": step_gbs, "algorithmic_bytes_per_step": algo_step,
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
-                         "traffic": profiled_traffic(dom, wl.layers) if wl.d == 8192 else None,
+                         "traffic": (profiled_traffic(dom, wl.layers)
+                                     if (wl.d == 8192 and args.path == "refresh" and args.layout == "rows"
+                                         and args.dtype == "bf16") else None),
                          "algorithmic_bytes": dom_bytes, "kernel_ms": dom_ms},
             "kernels_ms_per_step": kern_ms,
             "gpu_launches": nl * K,

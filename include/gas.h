@@ -73,7 +73,10 @@ typedef enum {
  * Create a handle for one model shape (the paper's Section 4 cost model
  * O(n_q * d_h * d) per layer per iteration).
  *   layers >= 1; d >= 8 and d % 8 == 0 (16-byte rows); n_q, n_kv >= 1 with
- *   n_q % n_kv == 0; d_h in {64, 128}; group size n_q/n_kv <= 64 (d_h 128) or 32 (d_h 64).
+ *   n_q % n_kv == 0; d_h in {64, 80, 96, 128, 256}; for d_h 64 / 128 the group size
+ *   n_q/n_kv <= 64 (d_h 128) or 32 (d_h 64).  The tensor-core back ends (fused, gram)
+ *   need d_h 64 or 128 and 16-bit weights; other head widths and fp32 weights run on
+ *   the streaming back end, which GAS_METHOD_AUTO then selects.
  * Allocates the device workspace on the current device (see gas_workspace_bytes).
  * Errors: GAS_ERR_INVALID_ARG (out == NULL, non-positive sizes), GAS_ERR_UNSUPPORTED
  * (shape limits above), GAS_ERR_ALLOC, GAS_ERR_CUDA.  *out is NULL on error.
@@ -170,13 +173,15 @@ gas_status gas_resolve_calibration(gas_handle h, double gamma, double delta_star
 #define GAS_DTYPE_F16  2
 
 /*
- * Weight element type: GAS_DTYPE_BF16 (default) or GAS_DTYPE_F16 (IEEE binary16).  With
- * binary16 weights the tensor-core operands (weights, and the hi + lo split start and
- * write-back vectors) are binary16 too; sigma and v keep the same fp32 accumulation.
- * The write-back's y / ||v'|| operand must lie inside binary16's range, which holds
- * unless ||W^K_g||_2 is below about 2^-14.  Host only; applies to later calls.
- * GAS_DTYPE_F32 -> GAS_ERR_UNSUPPORTED; anything else -> GAS_ERR_INVALID_ARG.
- * gas_spectral_norms_static always reads bf16.
+ * Weight element type: GAS_DTYPE_BF16 (default), GAS_DTYPE_F16 (IEEE binary16) or
+ * GAS_DTYPE_F32.  With binary16 weights the tensor-core operands (weights, and the
+ * hi + lo split start and write-back vectors) are binary16 too; sigma and v keep the
+ * same fp32 accumulation.  The write-back's y / ||v'|| operand must lie inside binary16's
+ * range, which holds unless ||W^K_g||_2 is below about 2^-14.  fp32 weights are read by
+ * the streaming back end and the whole-layer path only (d_h <= 128); AUTO selects the
+ * streaming back end for them, and the fused / gram back ends return
+ * GAS_ERR_UNSUPPORTED.  Host only; applies to later calls.  Unknown values ->
+ * GAS_ERR_INVALID_ARG.  gas_spectral_norms_static always reads bf16.
  */
 gas_status gas_set_weight_dtype(gas_handle h, int dtype);
 

@@ -157,7 +157,7 @@ def _ptr_array(tensors: Sequence[torch.Tensor], rows: int, d: int, name: str, la
             else:
                 heads, dh, ld, hs = layout
                 last = (heads - 1) * hs + (dh - 1) * ld + d - 1
-            avail = t.untyped_storage().nbytes() // 2 - t.storage_offset()
+            avail = t.untyped_storage().nbytes() // t.element_size() - t.storage_offset()
             if last >= avail:
                 raise ValueError(f"{name}[{i}]: the strided matrix needs {last + 1} elements, "
                                  f"the tensor's storage holds {avail} from its first element")
@@ -236,7 +236,7 @@ class Handle:
         code = {"bf16": GAS_DTYPE_BF16, torch.bfloat16: GAS_DTYPE_BF16, "f16": GAS_DTYPE_F16,
                 torch.float16: GAS_DTYPE_F16, "f32": GAS_DTYPE_F32, torch.float32: GAS_DTYPE_F32}[dtype]
         _check(load().gas_set_weight_dtype(self._h, code), self._h)
-        self._wdtype = torch.float16 if code == GAS_DTYPE_F16 else torch.bfloat16
+        self._wdtype = {GAS_DTYPE_F16: torch.float16, GAS_DTYPE_F32: torch.float32}.get(code, torch.bfloat16)
 
     def _weights(self, wq, wk):
         lq, lk = getattr(self, "_lq", None), getattr(self, "_lk", None)

@@ -359,7 +359,13 @@ gas_status spectral_impl(gas_ctx* h, const void* const* wq, const void* const* w
   gas::LayerTable tab;
   std::memset(&tab, 0, sizeof(tab));
   fill_table(h, tab, wq, wk);
-  const int method = h->method == GAS_METHOD_AUTO ? GAS_METHOD_FUSED : h->method;
+  const bool tc_ok = h->s.tc && !h->s.f32;
+  const int method = h->method == GAS_METHOD_AUTO ? (tc_ok ? GAS_METHOD_FUSED : GAS_METHOD_STREAM) : h->method;
+  if (method != GAS_METHOD_STREAM && !tc_ok)
+    return fail(h, GAS_ERR_UNSUPPORTED, "the tensor-core back ends need d_h 64 or 128 and 16-bit weights "
+                                        "(use GAS_METHOD_STREAM or AUTO)");
+  if (method == GAS_METHOD_STREAM && h->s.f32 && h->s.dh > 128)
+    return fail(h, GAS_ERR_UNSUPPORTED, "fp32 weights are supported up to d_h 128");
   if (method == GAS_METHOD_STREAM && h->s.cols)
     return fail(h, GAS_ERR_UNSUPPORTED, "the streaming back end reads the nn.Linear layout only (use fused or gram)");
   if (method == GAS_METHOD_STREAM) return run_stream(h, tab, iters, v_in, v_out, sigma, s_out, scale_c, st);
@@ -454,11 +460,15 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
     return fail(nullptr, GAS_ERR_UNSUPPORTED, "at most %d layers per handle", gas::kMaxLayers);
   if (d % 8 != 0 || d < 8) return fail(nullptr, GAS_ERR_UNSUPPORTED, "d must be a multiple of 8 (got %d)", d);
   if (n_q % n_kv != 0) return fail(nullptr, GAS_ERR_UNSUPPORTED, "n_q (%d) must be a multiple of n_kv (%d)", n_q, n_kv);
-  if (d_h != 64 && d_h != 128) return fail(nullptr, GAS_ERR_UNSUPPORTED, "d_h must be 64 or 128 (got %d)", d_h);
+  if (d_h != 64 && d_h != 80 && d_h != 96 && d_h != 128 && d_h != 256)
+    return fail(nullptr, GAS_ERR_UNSUPPORTED, "d_h must be 64, 80, 96, 128 or 256 (got %d)", d_h);
   const int G = n_q / n_kv;
-  const int gpt = 128 / d_h;
+  // d_h 64 / 128: whole heads fill 128-row tiles and the tensor-core back ends apply;
+  // other head widths run on the streaming back end only.
+  const bool tc = d_h == 64 || d_h == 128;
+  const int gpt = tc ? 128 / d_h : 1;
   const int nz = round_up16(2 * G * gpt);
-  if (nz > 128)
+  if (tc && nz > 128)
     return fail(nullptr, GAS_ERR_UNSUPPORTED, "group size %d too large for d_h %d (max %d)", G, d_h, 64 / gpt);
   int nz_t = nz <= 16 ? 16 : nz <= 32 ? 32 : nz <= 64 ? 64 : 128;
 
@@ -475,6 +485,8 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   s.hsq = s.hsk = static_cast<long long>(d_h) * d;
   s.f16 = 0;
   s.cols = 0;
+  s.f32 = 0;
+  s.tc = tc ? 1 : 0;
 
   cudaError_t e = cudaGetDevice(&h->device);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
@@ -486,7 +498,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
     delete h;
     return st;
   }
-  if (cc_major != 10 || static_cast<size_t>(smem_optin) < gas::gram_smem_bytes(s.nz)) {
+  if (cc_major != 10 || (tc && static_cast<size_t>(smem_optin) < gas::gram_smem_bytes(s.nz))) {
     delete h;
     return fail(nullptr, GAS_ERR_UNSUPPORTED, "needs an sm_10x GPU with >= %zu B shared memory per block",
                 gas::gram_smem_bytes(s.nz));
@@ -630,11 +642,10 @@ gas_status gas_set_weight_layout(gas_handle h, int layout, long long ld_q, long 
 
 gas_status gas_set_weight_dtype(gas_handle h, int dtype) {
   if (!h) return GAS_ERR_INVALID_ARG;
-  if (dtype == GAS_DTYPE_F32)
-    return fail(h, GAS_ERR_UNSUPPORTED, "fp32 weights are not implemented (bf16 or fp16 only)");
-  if (dtype != GAS_DTYPE_BF16 && dtype != GAS_DTYPE_F16)
+  if (dtype != GAS_DTYPE_BF16 && dtype != GAS_DTYPE_F16 && dtype != GAS_DTYPE_F32)
     return fail(h, GAS_ERR_INVALID_ARG, "unknown weight dtype %d", dtype);
   h->s.f16 = dtype == GAS_DTYPE_F16 ? 1 : 0;
+  h->s.f32 = dtype == GAS_DTYPE_F32 ? 1 : 0;
   return GAS_OK;
 }
 

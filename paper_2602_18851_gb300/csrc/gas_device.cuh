@@ -42,6 +42,50 @@ __device__ __forceinline__ void unpack8w(const uint4& q, float (&f)[8]) {
   else unpack8(q, f);
 }
 
+// Weight element types of the CUDA-core kernels: bf16, binary16, fp32.
+enum WeightType : int { kWBf16 = 0, kWF16 = 1, kWF32 = 2 };
+
+// Eight consecutive weights (16 bytes of 16-bit values, 32 bytes of fp32) as loaded.
+template <int WT>
+struct W8 {
+  uint4 q[WT == kWF32 ? 2 : 1];
+};
+
+// Streaming (evict-first) load of the eight weights at element offset `off` of `base`.
+template <int WT>
+__device__ __forceinline__ W8<WT> load_w8(const void* base, long long off) {
+  W8<WT> w;
+  if (WT == kWF32) {
+    const uint4* p = reinterpret_cast<const uint4*>(static_cast<const float*>(base) + off);
+    w.q[0] = __ldcs(p);
+    w.q[1] = __ldcs(p + 1);
+  } else {
+    w.q[0] = __ldcs(reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(base) + off));
+  }
+  return w;
+}
+
+template <int WT>
+__device__ __forceinline__ W8<WT> zero_w8() {
+  W8<WT> w;
+#pragma unroll
+  for (int i = 0; i < (WT == kWF32 ? 2 : 1); ++i) w.q[i] = make_uint4(0, 0, 0, 0);
+  return w;
+}
+
+template <int WT>
+__device__ __forceinline__ void unpack_w8(const W8<WT>& w, float (&f)[8]) {
+  if (WT == kWBf16) {
+    unpack8(w.q[0], f);
+  } else if (WT == kWF16) {
+    unpack8_f16(w.q[0], f);
+  } else {
+    const uint32_t b[8] = {w.q[0].x, w.q[0].y, w.q[0].z, w.q[0].w, w.q[1].x, w.q[1].y, w.q[1].z, w.q[1].w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) f[i] = __uint_as_float(b[i]);
+  }
+}
+
 // Round-to-nearest-even fp32 -> bf16 bits.
 __device__ __forceinline__ uint32_t f32_to_bf16_bits(float x) {
   return static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(x)));

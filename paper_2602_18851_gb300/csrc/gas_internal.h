@@ -37,6 +37,8 @@ struct Shape {
   long long hsk;  // elements between the first rows of consecutive key groups (>= d_h * ldk)
   int f16;        // weights (and the MMA operands) are binary16 instead of bf16
   int cols;       // GPT-2 Conv1D layout: element (row r, column c) at w[c * ld + r]
+  int f32;        // fp32 weights (CUDA-core back ends only)
+  int tc;         // d_h in {64, 128}: the tensor-core back ends apply
 };
 
 // Element offset of row r (head r / d_h, row r % d_h inside it) of a weight matrix.

@@ -44,7 +44,7 @@ __device__ __forceinline__ void stage_vector(float* xs, const float* src, int n,
 }
 
 // out[l][r] = sum_c W_l[r][c] * x_l[c] for a block of 64 rows; x = src/||src|| (d values).
-template <bool F16>
+template <int WT>
 __global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant__ LayerTable tab,
                                                            const __grid_constant__ LayerArgs a) {
   extern __shared__ float lsm[];
@@ -53,7 +53,7 @@ __global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant
   const int l = blockIdx.y;
   const bool isq = a.which == 1;
   const int R = (isq ? a.s.nq : a.s.nkv) * a.s.dh;
-  const uint16_t* W = isq ? tab.q[l] : tab.k[l];
+  const void* W = isq ? tab.q[l] : tab.k[l];
   const long long ld = isq ? a.s.ldq : a.s.ldk;
   const long long hstride = isq ? a.s.hsq : a.s.hsk;
   stage_vector(xs, a.src + static_cast<size_t>(l) * a.s.d, a.s.d, 1, red);
@@ -69,10 +69,9 @@ __global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       if (r0 + i < R) {
-        const uint4 q =
-            __ldcs(reinterpret_cast<const uint4*>(W + weight_row_offset(r0 + i, a.s.dh, ld, hstride) + c));
+        const W8<WT> q = load_w8<WT>(W, weight_row_offset(r0 + i, a.s.dh, ld, hstride) + c);
         float f[8];
-        unpack8w<F16>(q, f);
+        unpack_w8<WT>(q, f);
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc[i] = fmaf(f[e], xv[e], acc[i]);
       }
@@ -86,7 +85,7 @@ __global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant
 
 // out[l][c] = sum_r W_l[r][c] * x_l[r] for a chunk of 256 columns over all rows, with
 // x = RepeatBlocks(src) (query matrix) or SumGroups(src) (key matrix).
-template <bool F16>
+template <int WT>
 __global__ void __launch_bounds__(256) layer_coldot_kernel(const __grid_constant__ LayerTable tab,
                                                            const __grid_constant__ LayerArgs a) {
   extern __shared__ float lsm[];
@@ -94,7 +93,7 @@ __global__ void __launch_bounds__(256) layer_coldot_kernel(const __grid_constant
   const int l = blockIdx.y;
   const bool isq = a.which == 1;
   const int R = (isq ? s.nq : s.nkv) * s.dh;
-  const uint16_t* W = isq ? tab.q[l] : tab.k[l];
+  const void* W = isq ? tab.q[l] : tab.k[l];
   const long long ld = isq ? s.ldq : s.ldk;
   const long long hstride = isq ? s.hsq : s.hsk;
   float* xs = lsm;                  // [R]
@@ -121,9 +120,9 @@ __global__ void __launch_bounds__(256) layer_coldot_kernel(const __grid_constant
   if (c < s.d) {
 #pragma unroll 4
     for (int r = warp; r < R; r += 8) {
-      const uint4 q = __ldcs(reinterpret_cast<const uint4*>(W + weight_row_offset(r, s.dh, ld, hstride) + c));
+      const W8<WT> q = load_w8<WT>(W, weight_row_offset(r, s.dh, ld, hstride) + c);
       float f[8];
-      unpack8w<F16>(q, f);
+      unpack_w8<WT>(q, f);
       const float xr = xs[r];
 #pragma unroll
       for (int e = 0; e < 8; ++e) acc[e] = fmaf(f[e], xr, acc[e]);
@@ -189,40 +188,42 @@ __global__ void __launch_bounds__(256) layer_finalize_kernel(const __grid_consta
 
 }  // namespace
 
-template <bool F16>
+template <int WT>
 cudaError_t launch_rowdot_dt(const LayerTable& tab, const LayerArgs& a, cudaStream_t st) {
   const int R = (a.which == 1 ? a.s.nq : a.s.nkv) * a.s.dh;
   const dim3 grid((R + kRowBlock - 1) / kRowBlock, a.s.L);
   const size_t smem = (a.s.d + 8) * sizeof(float);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(layer_rowdot_kernel<F16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(layer_rowdot_kernel<WT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
-  layer_rowdot_kernel<F16><<<grid, 256, smem, st>>>(tab, a);
+  layer_rowdot_kernel<WT><<<grid, 256, smem, st>>>(tab, a);
   return cudaGetLastError();
 }
 
-template <bool F16>
+template <int WT>
 cudaError_t launch_coldot_dt(const LayerTable& tab, const LayerArgs& a, cudaStream_t st) {
   const int R = (a.which == 1 ? a.s.nq : a.s.nkv) * a.s.dh;
   const dim3 grid((a.s.d + 255) / 256, a.s.L);
   const size_t smem = (R + 8 * 256) * sizeof(float);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(layer_coldot_kernel<F16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(layer_coldot_kernel<WT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
-  layer_coldot_kernel<F16><<<grid, 256, smem, st>>>(tab, a);
+  layer_coldot_kernel<WT><<<grid, 256, smem, st>>>(tab, a);
   return cudaGetLastError();
 }
 
 cudaError_t launch_layer_rowdot(const LayerTable& tab, const LayerArgs& a, cudaStream_t st) {
-  return a.s.f16 ? launch_rowdot_dt<true>(tab, a, st) : launch_rowdot_dt<false>(tab, a, st);
+  return a.s.f32 ? launch_rowdot_dt<kWF32>(tab, a, st)
+                 : a.s.f16 ? launch_rowdot_dt<kWF16>(tab, a, st) : launch_rowdot_dt<kWBf16>(tab, a, st);
 }
 
 cudaError_t launch_layer_coldot(const LayerTable& tab, const LayerArgs& a, cudaStream_t st) {
-  return a.s.f16 ? launch_coldot_dt<true>(tab, a, st) : launch_coldot_dt<false>(tab, a, st);
+  return a.s.f32 ? launch_coldot_dt<kWF32>(tab, a, st)
+                 : a.s.f16 ? launch_coldot_dt<kWF16>(tab, a, st) : launch_coldot_dt<kWBf16>(tab, a, st);
 }
 
 cudaError_t launch_layer_finalize(const LayerArgs& a, cudaStream_t st) {

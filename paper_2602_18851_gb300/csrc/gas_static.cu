@@ -82,6 +82,8 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
   s.ldq = s.ldk = d;
   s.hsq = s.hsk = static_cast<long long>(d_h) * d;
   s.f16 = 0;
+  s.f32 = 0;
+  s.tc = 1;
   // Scratch: z and t partials [L][n_q][nch][d_h], their squared-norm partials [L][n_q][nch].
   const size_t vec = static_cast<size_t>(layers) * n_q * s.nch * d_h * sizeof(float);
   const size_t nrm = static_cast<size_t>(layers) * n_q * s.nch * sizeof(float);

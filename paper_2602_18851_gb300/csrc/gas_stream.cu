@@ -7,7 +7,8 @@
 // (z = B_g v for the normalised v, so z_next must be divided by ||v'||; the consumer
 // does that when it sums the partials).  The start is a K0 pass z = B_g v_in with
 // ||v_in||^2, and the last K pass writes v' itself (normalised by the finalize kernel).
-// Each CTA streams one d_h x 256 bf16 tile with 16-byte loads; partial results over
+// Each CTA streams one d_h x 256 weight tile (bf16, binary16 or fp32; any d_h in
+// {64, 80, 96, 128, 256}) with 16-byte loads; partial results over
 // its columns go to a small fp32 workspace indexed by chunk and are summed, in a fixed
 // order, by the next pass (no atomics, deterministic).
 
@@ -17,14 +18,18 @@ namespace gas {
 
 namespace {
 
-__device__ __forceinline__ uint4 load_stream16(const uint16_t* p) {
-  return __ldcs(reinterpret_cast<const uint4*>(p));
-}
+// Smallest power of two >= x (the warp transpose-reduction works on 2^n values).
+__host__ __device__ constexpr int pow2_at_least(int x) { return x <= 1 ? 1 : 2 * pow2_at_least((x + 1) / 2); }
 
-template <int DH, int MODE, bool F16>
-__global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant__ LayerTable tab,
-                                                          const __grid_constant__ StreamArgs a) {
-  constexpr int R = DH / 8;  // rows held per thread (warp w owns rows w, w+8, ...)
+// Warps per CTA: 8, or 16 for d_h 256 so that every thread holds at most 16 rows.
+__host__ __device__ constexpr int stream_warps(int dh) { return dh > 128 ? 16 : 8; }
+
+template <int DH, int MODE, int WT>
+__global__ void __launch_bounds__(32 * stream_warps(DH)) stream_pass_kernel(const __grid_constant__ LayerTable tab,
+                                                                            const __grid_constant__ StreamArgs a) {
+  constexpr int NW = stream_warps(DH);
+  constexpr int RV = DH / NW;             // rows held per thread (warp w owns rows w, w+NW, ...)
+  constexpr int R = pow2_at_least(RV);    // padded to a power of two with zero rows
   const Shape& s = a.s;
   const int chunk = blockIdx.x, m = blockIdx.y, l = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -32,17 +37,18 @@ __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant_
   const bool colok = col < s.d;  // d % 8 == 0: a lane's 8 columns are all in or all out
   const long long ld = (MODE == kPassQ) ? s.ldq : s.ldk;
   const long long hstride = (MODE == kPassQ) ? s.hsq : s.hsk;
-  const uint16_t* X = ((MODE == kPassQ) ? tab.q[l] : tab.k[l]) + static_cast<size_t>(m) * hstride;
+  const void* X = (MODE == kPassQ) ? tab.q[l] : tab.k[l];
+  const long long x0 = static_cast<long long>(m) * hstride;
 
-  uint4 w[R];
+  W8<WT> w[R];
 #pragma unroll
   for (int rr = 0; rr < R; ++rr) {
-    const int row = warp + 8 * rr;
-    w[rr] = colok ? load_stream16(X + static_cast<size_t>(row) * ld + col) : make_uint4(0, 0, 0, 0);
+    const int row = warp + NW * rr;
+    w[rr] = (rr < RV && colok) ? load_w8<WT>(X, x0 + static_cast<long long>(row) * ld + col) : zero_w8<WT>();
   }
 
   __shared__ float xs[DH];
-  __shared__ __align__(16) float red[8][kStreamChunk];
+  __shared__ __align__(16) float red[NW][kStreamChunk];
   __shared__ __align__(16) float ps[kStreamChunk];
 
   const int nvec = (MODE == kPassQ) ? 1 : s.G;
@@ -77,10 +83,10 @@ __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant_
 #pragma unroll
       for (int c = 0; c < 8; ++c) pp[c] = 0.0f;
 #pragma unroll
-      for (int rr = 0; rr < R; ++rr) {
+      for (int rr = 0; rr < RV; ++rr) {
         float f[8];
-        unpack8w<F16>(w[rr], f);
-        const float xr = xs[warp + 8 * rr];
+        unpack_w8<WT>(w[rr], f);
+        const float xr = xs[warp + NW * rr];
 #pragma unroll
         for (int c = 0; c < 8; ++c) pp[c] = fmaf(f[c], xr, pp[c]);
       }
@@ -89,9 +95,10 @@ __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant_
       rp[1] = make_float4(pp[4], pp[5], pp[6], pp[7]);
       __syncthreads();
       float tot = 0.0f;
-#pragma unroll
-      for (int ww = 0; ww < 8; ++ww) tot += red[ww][tid];
-      ps[tid] = tot;
+      if (tid < kStreamChunk) {
+        for (int ww = 0; ww < NW; ++ww) tot += red[ww][tid];
+        ps[tid] = tot;
+      }
       __syncthreads();
       const float4* pq = reinterpret_cast<const float4*>(&ps[lane * 8]);
       const float4 p0 = pq[0], p1 = pq[1];
@@ -116,7 +123,7 @@ __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant_
 #pragma unroll
       for (int rr = 0; rr < R; ++rr) {
         float f[8];
-        unpack8w<F16>(w[rr], f);
+        unpack_w8<WT>(w[rr], f);
         float acc = 0.0f;
 #pragma unroll
         for (int c = 0; c < 8; ++c) acc = fmaf(f[c], p[c], acc);
@@ -124,8 +131,8 @@ __global__ void __launch_bounds__(256) stream_pass_kernel(const __grid_constant_
       }
       int idx;
       const float r = warp_transpose_reduce<R>(qv, lane, idx);
-      if (transpose_reduce_writer<R>(lane))
-        a.out[(hidx * s.nch + chunk) * DH + warp + 8 * idx] = r;
+      if (transpose_reduce_writer<R>(lane) && idx < RV)
+        a.out[(hidx * s.nch + chunk) * DH + warp + NW * idx] = r;
     }
   }
   if (MODE == kPassK0 && a.s_zero != nullptr && chunk == 0 && m == 0 && tid == 0) a.s_zero[l] = 0.0f;
@@ -169,15 +176,15 @@ __global__ void __launch_bounds__(32) scales_kernel(const __grid_constant__ Scal
   if (threadIdx.x == 0) a.s[l] = a.scale_c * m;
 }
 
-template <int DH, bool F16>
+template <int DH, int WT>
 cudaError_t launch_stream_dt(const LayerTable& tab, const StreamArgs& a, cudaStream_t st) {
-  const dim3 block(256);
+  const dim3 block(32 * stream_warps(DH));
   const dim3 grid(a.s.nch, a.mode == kPassQ ? a.s.nq : a.s.nkv, a.s.L);
   switch (a.mode) {
-    case kPassQ: stream_pass_kernel<DH, kPassQ, F16><<<grid, block, 0, st>>>(tab, a); break;
-    case kPassK: stream_pass_kernel<DH, kPassK, F16><<<grid, block, 0, st>>>(tab, a); break;
-    case kPassK0: stream_pass_kernel<DH, kPassK0, F16><<<grid, block, 0, st>>>(tab, a); break;
-    case kPassKOut: stream_pass_kernel<DH, kPassKOut, F16><<<grid, block, 0, st>>>(tab, a); break;
+    case kPassQ: stream_pass_kernel<DH, kPassQ, WT><<<grid, block, 0, st>>>(tab, a); break;
+    case kPassK: stream_pass_kernel<DH, kPassK, WT><<<grid, block, 0, st>>>(tab, a); break;
+    case kPassK0: stream_pass_kernel<DH, kPassK0, WT><<<grid, block, 0, st>>>(tab, a); break;
+    case kPassKOut: stream_pass_kernel<DH, kPassKOut, WT><<<grid, block, 0, st>>>(tab, a); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
@@ -185,15 +192,24 @@ cudaError_t launch_stream_dt(const LayerTable& tab, const StreamArgs& a, cudaStr
 
 template <int DH>
 cudaError_t launch_stream_dh(const LayerTable& tab, const StreamArgs& a, cudaStream_t st) {
-  return a.s.f16 ? launch_stream_dt<DH, true>(tab, a, st) : launch_stream_dt<DH, false>(tab, a, st);
+  if (a.s.f32) {
+    if (DH > 128) return cudaErrorInvalidValue;  // fp32 rows of d_h 256 do not fit the registers
+    return launch_stream_dt<(DH > 128 ? 128 : DH), kWF32>(tab, a, st);
+  }
+  return a.s.f16 ? launch_stream_dt<DH, kWF16>(tab, a, st) : launch_stream_dt<DH, kWBf16>(tab, a, st);
 }
 
 }  // namespace
 
 cudaError_t launch_stream_pass(const LayerTable& tab, const StreamArgs& a, cudaStream_t st) {
-  if (a.s.dh == 128) return launch_stream_dh<128>(tab, a, st);
-  if (a.s.dh == 64) return launch_stream_dh<64>(tab, a, st);
-  return cudaErrorInvalidValue;
+  switch (a.s.dh) {
+    case 64: return launch_stream_dh<64>(tab, a, st);
+    case 80: return launch_stream_dh<80>(tab, a, st);
+    case 96: return launch_stream_dh<96>(tab, a, st);
+    case 128: return launch_stream_dh<128>(tab, a, st);
+    case 256: return launch_stream_dh<256>(tab, a, st);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st) {

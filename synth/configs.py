@@ -75,6 +75,11 @@ WORKLOADS = {
     # widest z0 / write-back operand, 128 rows).
     "tiny-g16": Workload("tiny-g16", 2, 384, 16, 1, 128, 8, "spike4", _BASE_SEED + 16),
     "tiny-g32": Workload("tiny-g32", 2, 320, 32, 1, 64, 8, "spike4", _BASE_SEED + 17),
+    # Head widths outside {64, 128} (streaming back end): 80 and 96 as in several
+    # published models, 256 as in wide-head ones.
+    "tiny-dh80": Workload("tiny-dh80", 2, 320, 4, 2, 80, 10, "spike4", _BASE_SEED + 18),
+    "tiny-dh96": Workload("tiny-dh96", 2, 384, 6, 3, 96, 10, "lognormal", _BASE_SEED + 19),
+    "tiny-dh256": Workload("tiny-dh256", 2, 512, 4, 2, 256, 10, "spike1", _BASE_SEED + 20),
 }
 
 # Transient recipe (per step, per weight matrix W of one head or KV group):

@@ -82,8 +82,8 @@ def test_weight_dtype_errors():
     wl = get_workload("tiny-gqa128")
     with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
         lib = gas.load()
-        assert lib.gas_set_weight_dtype(h._h, gas.GAS_DTYPE_F32) == gas.GAS_ERR_UNSUPPORTED
         assert lib.gas_set_weight_dtype(h._h, 7) == gas.GAS_ERR_INVALID_ARG
+        assert lib.gas_set_weight_dtype(h._h, gas.GAS_DTYPE_BF16) == gas.GAS_OK
         wq, wk, v_in = _inputs(wl)
         with pytest.raises(ValueError):
             h.refresh(wq, wk, 2, v_in)  # binary16 tensors on a bf16 handle
