@@ -40,6 +40,11 @@ struct gas_ctx {
   float* n2p = nullptr;   // [L][nq][nch]
   float* tp = nullptr;    // [L][nq][nch][dh]
   float* s2p = nullptr;   // [L][nq][nch]
+  float* zr = nullptr;    // [L][nq][dh]  chunk sums of the streaming passes
+  float* n2r = nullptr;   // [L][nq]
+  float* tr = nullptr;    // [L][nq][dh]
+  float* s2r = nullptr;   // [L][nq]
+  unsigned* tickets = nullptr;  // [L][nq] last-CTA counters of the streaming passes
   uint16_t* vhl = nullptr;
   float* gq = nullptr;
   float* gk = nullptr;
@@ -223,6 +228,9 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
   a.mode = gas::kPassK0;
   a.out = h->zp;
   a.out2 = h->n2p;
+  a.outr = h->zr;
+  a.outr2 = h->n2r;
+  a.tickets = h->tickets;
   a.v_in = v_in;
   a.s_zero = s_out;
   cudaError_t e = launch(h, "stream_pass_k0", st, [&] { return gas::launch_stream_pass(tab, a, st); });
@@ -231,12 +239,14 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
     gas::StreamArgs q{};
     q.s = s;
     q.mode = gas::kPassQ;
-    q.in_nch = s.nch;
     q.in_scaled = 1;
-    q.in = h->zp;
-    q.in2 = h->n2p;
+    q.in = h->zr;
+    q.in2 = h->n2r;
     q.out = h->tp;
     q.out2 = h->s2p;
+    q.outr = h->tr;
+    q.outr2 = h->s2r;
+    q.tickets = h->tickets;
     e = launch(h, "stream_pass_q", st, [&] { return gas::launch_stream_pass(tab, q, st); });
     ++launches;
     if (e != cudaSuccess) break;
@@ -245,12 +255,14 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
     gas::StreamArgs k{};
     k.s = s;
     k.mode = last ? gas::kPassKOut : gas::kPassK;
-    k.in_nch = s.nch;
     k.in_scaled = 1;
-    k.in = h->tp;
-    k.in2 = h->s2p;
+    k.in = h->tr;
+    k.in2 = h->s2r;
     k.out = h->zp;
     k.out2 = h->n2p;
+    k.outr = h->zr;
+    k.outr2 = h->n2r;
+    k.tickets = h->tickets;
     k.v_out = v_out;
     e = launch(h, last ? "stream_pass_kout" : "stream_pass_k", st,
                [&] { return gas::launch_stream_pass(tab, k, st); });
@@ -259,8 +271,8 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
   if (e == cudaSuccess) {
     gas::FinalizeArgs f{};
     f.s = s;
-    f.s2p = h->s2p;
-    f.n2p = h->n2p;
+    f.s2 = h->s2r;
+    f.n2 = h->n2r;
     f.v_out = v_out;
     f.sigma = sigma;
     f.scale_out = s_out;
@@ -516,6 +528,11 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_n2p = take(L * NQ * NCH * 4);
   const size_t o_tp = take(L * NQ * NCH * DH * 4);
   const size_t o_s2p = take(L * NQ * NCH * 4);
+  const size_t o_zr = take(L * NQ * DH * 4);
+  const size_t o_n2r = take(L * NQ * 4);
+  const size_t o_tr = take(L * NQ * DH * 4);
+  const size_t o_s2r = take(L * NQ * 4);
+  const size_t o_tickets = take(L * NQ * sizeof(unsigned));
   const size_t o_vhl = take(L * s.tiles_k * static_cast<size_t>(s.nz) * d * 2);
   const size_t o_gq = take(L * s.tiles_q * 16384ull * 4);
   const size_t o_gk = take(L * s.tiles_k * 16384ull * 4);
@@ -541,6 +558,11 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   h->n2p = reinterpret_cast<float*>(b + o_n2p);
   h->tp = reinterpret_cast<float*>(b + o_tp);
   h->s2p = reinterpret_cast<float*>(b + o_s2p);
+  h->zr = reinterpret_cast<float*>(b + o_zr);
+  h->n2r = reinterpret_cast<float*>(b + o_n2r);
+  h->tr = reinterpret_cast<float*>(b + o_tr);
+  h->s2r = reinterpret_cast<float*>(b + o_s2r);
+  h->tickets = reinterpret_cast<unsigned*>(b + o_tickets);
   h->vhl = reinterpret_cast<uint16_t*>(b + o_vhl);
   h->gq = reinterpret_cast<float*>(b + o_gq);
   h->gk = reinterpret_cast<float*>(b + o_gk);

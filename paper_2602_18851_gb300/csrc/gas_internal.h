@@ -49,10 +49,12 @@ __host__ __device__ inline long long weight_row_offset(int r, int dh, long long 
 // ---- streaming matvec-chain passes (Algorithm 2 applied literally) ---------------
 // One pass streams one weight matrix X (a head's A_h or a group's B_g, d_h x d) in
 // column chunks.  For every vector that uses X it forms p = X^T x over the chunk
-// (and ||p||^2), then either q = X p (partial over the chunk) or writes p out.
+// (and ||p||^2), then either q = X p (partial over the chunk) or writes p out.  The
+// last chunk CTA of every matrix sums the chunk partials (in chunk order) into one
+// d_h-vector and one squared norm per head, which the next pass reads.
 enum StreamMode : int {
-  kPassQ = 0,      // X = A_h, x = z from K partials; out: t = A_h u' partials, ||u'||^2
-  kPassK = 1,      // X = B_g, x = y from Q partials (G heads); out: z = B_g v', ||v'||^2
+  kPassQ = 0,      // X = A_h, x = z / ||v'|| (K results); out: t = A_h u', ||u'||^2
+  kPassK = 1,      // X = B_g, x = t / ||u'|| = y (Q results, G heads); out: z = B_g v', ||v'||^2
   kPassK0 = 2,     // X = B_g, p = v_in chunk (G heads); out: z = B_g v, ||v||^2
   kPassKOut = 3,   // X = B_g, x = y (G heads); writes p (= v') to v_out, ||v'||^2
 };
@@ -60,21 +62,23 @@ enum StreamMode : int {
 struct StreamArgs {
   Shape s;
   int mode;
-  int in_nch;         // number of partial chunks to sum for the input vector
-  int in_scaled;      // 1: x = sum(in) / sqrt(sum(in2)); 0: x = sum(in)
-  const float* in;    // [L][nq][in_nch][dh]
-  const float* in2;   // [L][nq][in_nch]
-  float* out;         // [L][nq][nch][dh] (q partials)      (modes Q, K, K0)
-  float* out2;        // [L][nq][nch]     (||p||^2 partials) (all modes)
-  const float* v_in;  // [L][nq][d]                          (mode K0)
-  float* v_out;       // [L][nq][d]                          (mode KOut)
+  int in_scaled;      // 1: x = in / sqrt(in2); 0: x = in
+  const float* in;    // [L][nq][dh] input vector of every head (modes Q, K, KOut)
+  const float* in2;   // [L][nq]     its squared norm
+  float* out;         // [L][nq][nch][dh] q partials                 (modes Q, K, K0)
+  float* out2;        // [L][nq][nch]     ||p||^2 partials            (all modes)
+  float* outr;        // [L][nq][dh]      q summed over the chunks    (modes Q, K, K0)
+  float* outr2;       // [L][nq]          ||p||^2 summed over the chunks (all modes)
+  unsigned* tickets;  // [L][nq] chunk counters of the last-CTA reduction; zero between passes
+  const float* v_in;  // [L][nq][d]                                   (mode K0)
+  float* v_out;       // [L][nq][d]                                   (mode KOut)
   float* s_zero;      // mode K0: per-layer scale slots zeroed for the fused epilogue
 };
 
 struct FinalizeArgs {
   Shape s;
-  const float* s2p;   // [L][nq][nch] ||u'||^2 partials of the last Q pass
-  const float* n2p;   // [L][nq][nch] ||v'||^2 partials of the last K pass (or null)
+  const float* s2;    // [L][nq] ||u'||^2 of the last Q pass
+  const float* n2;    // [L][nq] ||v'||^2 of the last K pass (or null)
   float* v_out;       // [L][nq][d] raw v' (normalised in place) or null
   float* sigma;       // [L][nq]
   float* scale_out;   // [L] fused scale (atomic max) or null

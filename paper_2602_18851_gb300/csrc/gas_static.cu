@@ -84,10 +84,14 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
   s.f16 = 0;
   s.f32 = 0;
   s.tc = 1;
-  // Scratch: z and t partials [L][n_q][nch][d_h], their squared-norm partials [L][n_q][nch].
+  // Scratch: z and t partials [L][n_q][nch][d_h], their squared-norm partials [L][n_q][nch],
+  // the chunk sums of both ([L][n_q][d_h] and [L][n_q]) and the passes' ticket counters.
   const size_t vec = static_cast<size_t>(layers) * n_q * s.nch * d_h * sizeof(float);
   const size_t nrm = static_cast<size_t>(layers) * n_q * s.nch * sizeof(float);
-  const size_t need = 2 * gas::align256(vec) + 2 * gas::align256(nrm);
+  const size_t rvec = static_cast<size_t>(layers) * n_q * d_h * sizeof(float);
+  const size_t rnrm = static_cast<size_t>(layers) * n_q * sizeof(float);
+  const size_t need = 2 * gas::align256(vec) + 2 * gas::align256(nrm) + 2 * gas::align256(rvec) +
+                      3 * gas::align256(rnrm);
   if (need > gas::kStaticScratchBytes) {
     snprintf(buf, sizeof(buf),
              "gas_spectral_norms_static: this shape needs %zu bytes of scratch, the static array holds %zu",
@@ -109,8 +113,16 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
   float* tp = reinterpret_cast<float*>(b + gas::align256(vec));
   float* n2p = reinterpret_cast<float*>(b + 2 * gas::align256(vec));
   float* s2p = reinterpret_cast<float*>(b + 2 * gas::align256(vec) + gas::align256(nrm));
+  char* r = b + 2 * gas::align256(vec) + 2 * gas::align256(nrm);
+  float* zr = reinterpret_cast<float*>(r);
+  float* tr = reinterpret_cast<float*>(r + gas::align256(rvec));
+  float* n2r = reinterpret_cast<float*>(r + 2 * gas::align256(rvec));
+  float* s2r = reinterpret_cast<float*>(r + 2 * gas::align256(rvec) + gas::align256(rnrm));
+  unsigned* tickets = reinterpret_cast<unsigned*>(r + 2 * gas::align256(rvec) + 2 * gas::align256(rnrm));
   // Every scratch element a pass reads was written earlier in the same call (each pass
-  // covers all heads, chunks and rows), so nothing has to be cleared between calls.
+  // covers all heads, chunks and rows), so nothing has to be cleared between calls.  The
+  // ticket counters start at zero (a device array is zero-initialised when the module
+  // loads) and every pass leaves them at zero again.
 
   gas::LayerTable tab;
   std::memset(&tab, 0, sizeof(tab));
@@ -124,38 +136,45 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
   a.mode = gas::kPassK0;
   a.out = zp;
   a.out2 = n2p;
+  a.outr = zr;
+  a.outr2 = n2r;
+  a.tickets = tickets;
   a.v_in = v_in;
   e = gas::launch_stream_pass(tab, a, st);
   for (int it = 0; it < iters && e == cudaSuccess; ++it) {
     gas::StreamArgs q{};
     q.s = s;
     q.mode = gas::kPassQ;
-    q.in_nch = s.nch;
     q.in_scaled = 1;
-    q.in = zp;
-    q.in2 = n2p;
+    q.in = zr;
+    q.in2 = n2r;
     q.out = tp;
     q.out2 = s2p;
+    q.outr = tr;
+    q.outr2 = s2r;
+    q.tickets = tickets;
     e = gas::launch_stream_pass(tab, q, st);
     const bool last = (it == iters - 1);
     if (e != cudaSuccess || (last && v_out == nullptr)) break;
     gas::StreamArgs k{};
     k.s = s;
     k.mode = last ? gas::kPassKOut : gas::kPassK;
-    k.in_nch = s.nch;
     k.in_scaled = 1;
-    k.in = tp;
-    k.in2 = s2p;
+    k.in = tr;
+    k.in2 = s2r;
     k.out = zp;
     k.out2 = n2p;
+    k.outr = zr;
+    k.outr2 = n2r;
+    k.tickets = tickets;
     k.v_out = v_out;
     e = gas::launch_stream_pass(tab, k, st);
   }
   if (e == cudaSuccess) {
     gas::FinalizeArgs f{};
     f.s = s;
-    f.s2p = s2p;
-    f.n2p = n2p;
+    f.s2 = s2r;
+    f.n2 = n2r;
     f.v_out = v_out;
     f.sigma = sigma;
     e = gas::launch_finalize(f, st);

@@ -4,13 +4,16 @@
 // One power iteration for head h (group g) is two weight passes:
 //   Q pass over A_h = (W^Q_h)^T:  u' = A_h^T z (per column chunk), ||u'||^2, t = A_h u'
 //   K pass over B_g = (W^K_g)^T:  y = t/||u'||;  v' = B_g^T y, ||v'||^2, z_next = B_g v'
-// (z = B_g v for the normalised v, so z_next must be divided by ||v'||; the consumer
-// does that when it sums the partials).  The start is a K0 pass z = B_g v_in with
+// (z = B_g v for the normalised v, so z_next must be divided by ||v'||; the next Q
+// pass does that when it reads it).  The start is a K0 pass z = B_g v_in with
 // ||v_in||^2, and the last K pass writes v' itself (normalised by the finalize kernel).
 // Each CTA streams one d_h x 256 weight tile (bf16, binary16 or fp32; any d_h in
-// {64, 80, 96, 128, 256}) with 16-byte loads; partial results over
-// its columns go to a small fp32 workspace indexed by chunk and are summed, in a fixed
-// order, by the next pass (no atomics, deterministic).
+// {64, 80, 96, 128, 256}) with 16-byte loads, issued before anything else, and stages
+// its input vectors (one, or the G of a key group) in shared memory while they land.
+// Its results over its columns go to a small fp32 workspace indexed by chunk; the last
+// CTA of each matrix to finish (a ticket counter) sums them in chunk order into one
+// d_h-vector and one squared norm per head.  No float atomics: results are
+// deterministic.
 
 #include "gas_device.cuh"
 
@@ -24,10 +27,16 @@ __host__ __device__ constexpr int pow2_at_least(int x) { return x <= 1 ? 1 : 2 *
 // Warps per CTA: 8, or 16 for d_h 256 so that every thread holds at most 16 rows.
 __host__ __device__ constexpr int stream_warps(int dh) { return dh > 128 ? 16 : 8; }
 
+constexpr int kStreamVB = 8;  // input vectors staged in shared memory at a time
+
+// Two CTAs per SM for 16-bit weights (one tile loading while the other reduces); fp32
+// tiles need twice the registers.
 template <int DH, int MODE, int WT>
-__global__ void __launch_bounds__(32 * stream_warps(DH)) stream_pass_kernel(const __grid_constant__ LayerTable tab,
+__global__ void __launch_bounds__(32 * stream_warps(DH), (WT == kWF32 || DH > 128) ? 1 : 2)
+    stream_pass_kernel(const __grid_constant__ LayerTable tab,
                                                                             const __grid_constant__ StreamArgs a) {
   constexpr int NW = stream_warps(DH);
+  constexpr int NT = 32 * NW;
   constexpr int RV = DH / NW;             // rows held per thread (warp w owns rows w, w+NW, ...)
   constexpr int R = pow2_at_least(RV);    // padded to a power of two with zero rows
   const Shape& s = a.s;
@@ -47,95 +56,135 @@ __global__ void __launch_bounds__(32 * stream_warps(DH)) stream_pass_kernel(cons
     w[rr] = (rr < RV && colok) ? load_w8<WT>(X, x0 + static_cast<long long>(row) * ld + col) : zero_w8<WT>();
   }
 
-  __shared__ float xs[DH];
+  __shared__ __align__(16) float xs[kStreamVB][DH];
   __shared__ __align__(16) float red[NW][kStreamChunk];
   __shared__ __align__(16) float ps[kStreamChunk];
+  __shared__ unsigned is_last;
 
   const int nvec = (MODE == kPassQ) ? 1 : s.G;
-  for (int j = 0; j < nvec; ++j) {
-    const int h = (MODE == kPassQ) ? m : m * s.G + j;
-    const size_t hidx = static_cast<size_t>(l) * s.nq + h;
-    float p[8];
-    if (MODE == kPassK0) {
-      if (colok) {
-        const float4* vp = reinterpret_cast<const float4*>(a.v_in + hidx * s.d + col);
-        const float4 v0 = __ldg(vp), v1 = __ldg(vp + 1);
-        p[0] = v0.x; p[1] = v0.y; p[2] = v0.z; p[3] = v0.w;
-        p[4] = v1.x; p[5] = v1.y; p[6] = v1.z; p[7] = v1.w;
-      } else {
-#pragma unroll
-        for (int c = 0; c < 8; ++c) p[c] = 0.0f;
+  const size_t h0 = static_cast<size_t>(l) * s.nq + ((MODE == kPassQ) ? m : m * s.G);  // head of vector 0
+  for (int j0 = 0; j0 < nvec; j0 += kStreamVB) {
+    const int nb = min(kStreamVB, nvec - j0);
+    if (MODE != kPassK0) {
+      if (j0 > 0) __syncthreads();  // every thread is done with the previous batch
+      for (int i = tid; i < nb * DH; i += NT) {
+        const int jj = i / DH, r = i - jj * DH;
+        const size_t hidx = h0 + j0 + jj;
+        float x = __ldg(a.in + hidx * DH + r);
+        if (a.in_scaled) x *= safe_inv_sqrt(__ldg(a.in2 + hidx));
+        xs[jj][r] = x;
       }
-    } else {
-      __syncthreads();  // every thread is done with xs / ps of the previous vector
-      if (tid < DH) {
-        float acc = 0.0f;
-        for (int ch = 0; ch < a.in_nch; ++ch) acc += a.in[(hidx * a.in_nch + ch) * DH + tid];
-        if (a.in_scaled) {
-          float n2 = 0.0f;
-          for (int ch = 0; ch < a.in_nch; ++ch) n2 += a.in2[hidx * a.in_nch + ch];
-          acc *= safe_inv_sqrt(n2);
+      __syncthreads();
+    }
+    for (int jj = 0; jj < nb; ++jj) {
+      const size_t hidx = h0 + j0 + jj;
+      float p[8];
+      if (MODE == kPassK0) {
+        if (colok) {
+          const float4* vp = reinterpret_cast<const float4*>(a.v_in + hidx * s.d + col);
+          const float4 v0 = __ldg(vp), v1 = __ldg(vp + 1);
+          p[0] = v0.x; p[1] = v0.y; p[2] = v0.z; p[3] = v0.w;
+          p[4] = v1.x; p[5] = v1.y; p[6] = v1.z; p[7] = v1.w;
+        } else {
+#pragma unroll
+          for (int c = 0; c < 8; ++c) p[c] = 0.0f;
         }
-        xs[tid] = acc;
-      }
-      __syncthreads();
-      float pp[8];
+      } else {
+        // p = X^T x over this chunk: per-warp partials over its rows, then summed
+        float pp[8];
 #pragma unroll
-      for (int c = 0; c < 8; ++c) pp[c] = 0.0f;
+        for (int c = 0; c < 8; ++c) pp[c] = 0.0f;
 #pragma unroll
-      for (int rr = 0; rr < RV; ++rr) {
-        float f[8];
-        unpack_w8<WT>(w[rr], f);
-        const float xr = xs[warp + NW * rr];
+        for (int rr = 0; rr < RV; ++rr) {
+          float f[8];
+          unpack_w8<WT>(w[rr], f);
+          const float xr = xs[jj][warp + NW * rr];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) pp[c] = fmaf(f[c], xr, pp[c]);
+          for (int c = 0; c < 8; ++c) pp[c] = fmaf(f[c], xr, pp[c]);
+        }
+        float4* rp = reinterpret_cast<float4*>(&red[warp][lane * 8]);
+        rp[0] = make_float4(pp[0], pp[1], pp[2], pp[3]);
+        rp[1] = make_float4(pp[4], pp[5], pp[6], pp[7]);
+        __syncthreads();
+        if (tid < kStreamChunk) {
+          float tot = 0.0f;
+          for (int ww = 0; ww < NW; ++ww) tot += red[ww][tid];
+          ps[tid] = tot;
+        }
+        __syncthreads();
+        const float4* pq = reinterpret_cast<const float4*>(&ps[lane * 8]);
+        const float4 p0 = pq[0], p1 = pq[1];
+        p[0] = p0.x; p[1] = p0.y; p[2] = p0.z; p[3] = p0.w;
+        p[4] = p1.x; p[5] = p1.y; p[6] = p1.z; p[7] = p1.w;
       }
-      float4* rp = reinterpret_cast<float4*>(&red[warp][lane * 8]);
-      rp[0] = make_float4(pp[0], pp[1], pp[2], pp[3]);
-      rp[1] = make_float4(pp[4], pp[5], pp[6], pp[7]);
-      __syncthreads();
-      float tot = 0.0f;
-      if (tid < kStreamChunk) {
-        for (int ww = 0; ww < NW; ++ww) tot += red[ww][tid];
-        ps[tid] = tot;
-      }
-      __syncthreads();
-      const float4* pq = reinterpret_cast<const float4*>(&ps[lane * 8]);
-      const float4 p0 = pq[0], p1 = pq[1];
-      p[0] = p0.x; p[1] = p0.y; p[2] = p0.z; p[3] = p0.w;
-      p[4] = p1.x; p[5] = p1.y; p[6] = p1.z; p[7] = p1.w;
-    }
 
-    if (warp == 0) {  // each warp's lanes span the whole chunk: warp 0 owns ||p||^2
-      float q2 = 0.0f;
+      if (warp == 0) {  // each warp's lanes span the whole chunk: warp 0 owns ||p||^2
+        float q2 = 0.0f;
 #pragma unroll
-      for (int c = 0; c < 8; ++c) q2 = fmaf(p[c], p[c], q2);
-      q2 = warp_sum(q2);
-      if (lane == 0) a.out2[hidx * s.nch + chunk] = q2;
-      if (MODE == kPassKOut && colok) {
-        float4* vo = reinterpret_cast<float4*>(a.v_out + hidx * s.d + col);
-        vo[0] = make_float4(p[0], p[1], p[2], p[3]);
-        vo[1] = make_float4(p[4], p[5], p[6], p[7]);
+        for (int c = 0; c < 8; ++c) q2 = fmaf(p[c], p[c], q2);
+        q2 = warp_sum(q2);
+        if (lane == 0) a.out2[hidx * s.nch + chunk] = q2;
+        if (MODE == kPassKOut && colok) {
+          float4* vo = reinterpret_cast<float4*>(a.v_out + hidx * s.d + col);
+          vo[0] = make_float4(p[0], p[1], p[2], p[3]);
+          vo[1] = make_float4(p[4], p[5], p[6], p[7]);
+        }
       }
-    }
-    if (MODE != kPassKOut) {
-      float qv[R];
+      if (MODE != kPassKOut) {
+        float qv[R];
 #pragma unroll
-      for (int rr = 0; rr < R; ++rr) {
-        float f[8];
-        unpack_w8<WT>(w[rr], f);
-        float acc = 0.0f;
+        for (int rr = 0; rr < R; ++rr) {
+          float f[8];
+          unpack_w8<WT>(w[rr], f);
+          float acc = 0.0f;
 #pragma unroll
-        for (int c = 0; c < 8; ++c) acc = fmaf(f[c], p[c], acc);
-        qv[rr] = acc;
+          for (int c = 0; c < 8; ++c) acc = fmaf(f[c], p[c], acc);
+          qv[rr] = acc;
+        }
+        int idx;
+        const float r = warp_transpose_reduce<R>(qv, lane, idx);
+        if (transpose_reduce_writer<R>(lane) && idx < RV)
+          a.out[(hidx * s.nch + chunk) * DH + warp + NW * idx] = r;
       }
-      int idx;
-      const float r = warp_transpose_reduce<R>(qv, lane, idx);
-      if (transpose_reduce_writer<R>(lane) && idx < RV)
-        a.out[(hidx * s.nch + chunk) * DH + warp + NW * idx] = r;
     }
   }
   if (MODE == kPassK0 && a.s_zero != nullptr && chunk == 0 && m == 0 && tid == 0) a.s_zero[l] = 0.0f;
+
+  // The last chunk CTA of this matrix sums every vector's chunk partials, in chunk order.
+  __threadfence();
+  __syncthreads();
+  unsigned* ticket = a.tickets + static_cast<size_t>(l) * gridDim.y + m;
+  if (tid == 0) is_last = (atomicAdd(ticket, 1u) + 1u == gridDim.x) ? 1u : 0u;
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  const int nch = s.nch;
+  if (MODE != kPassKOut) {
+    for (int i = tid; i < nvec * DH; i += NT) {
+      const int jj = i / DH, r = i - jj * DH;
+      const size_t hidx = h0 + jj;
+      const float* src = a.out + hidx * nch * DH + r;
+      float acc[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
+      for (int c0 = 0; c0 < nch; c0 += 8) {  // eight loads in flight per step
+        float t[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) t[e] = c0 + e < nch ? __ldcg(src + static_cast<size_t>(c0 + e) * DH) : 0.0f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] += t[e];
+      }
+      a.outr[hidx * DH + r] = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+    }
+  }
+  for (int jj = warp; jj < nvec; jj += NW) {
+    const size_t hidx = h0 + jj;
+    float v = 0.0f;
+    for (int c = lane; c < nch; c += 32) v += __ldcg(a.out2 + hidx * nch + c);
+    v = warp_sum(v);
+    if (lane == 0) a.outr2[hidx] = v;
+  }
+  if (tid == 0) *ticket = 0u;
 }
 
 // sigma = ||u'|| of the last Q pass; v_out = v' / ||v'|| of the last K pass; fused
@@ -144,12 +193,9 @@ __global__ void __launch_bounds__(256) finalize_kernel(const __grid_constant__ F
   const Shape& s = a.s;
   const size_t hidx = blockIdx.x;
   const int l = static_cast<int>(hidx / s.nq);
-  float s2 = 0.0f, n2 = 0.0f;
-  for (int ch = 0; ch < s.nch; ++ch) s2 += a.s2p[hidx * s.nch + ch];
-  const float sigma = sqrtf(s2);
+  const float sigma = sqrtf(a.s2[hidx]);
   if (a.v_out != nullptr) {
-    for (int ch = 0; ch < s.nch; ++ch) n2 += a.n2p[hidx * s.nch + ch];
-    const float inv = safe_inv_sqrt(n2);
+    const float inv = safe_inv_sqrt(a.n2[hidx]);
     float4* v = reinterpret_cast<float4*>(a.v_out + hidx * s.d);
     for (int i = threadIdx.x; i < s.d / 4; i += blockDim.x) {
       float4 x = v[i];
