@@ -34,10 +34,13 @@ constexpr uint32_t kTileBytes = 128u * 64u * 2u;  // one 128-row x 64-column bf1
 constexpr int kSmemBudget = 232448;               // 227 KB opt-in dynamic shared memory
 constexpr int kSmemReserve = 22528;               // alignment slack, barriers, epilogue scratch
 
-template <int NZ>
+// A ring stage holds BPS consecutive 64-column chunks of a tile: BPS weight boxes, then
+// (key tiles) the BPS matching v boxes.  Two chunks per stage halve the per-byte count of
+// barrier waits, commits and copy issues on the producer and MMA threads.
+template <int NZ, int BPS>
 struct GramCfg {
   static constexpr uint32_t kVBytes = static_cast<uint32_t>(NZ) * 64u * 2u;
-  static constexpr uint32_t kStageBytes = kTileBytes + kVBytes;
+  static constexpr uint32_t kStageBytes = BPS * (kTileBytes + kVBytes);
   static constexpr int kStages = (kSmemBudget - kSmemReserve) / static_cast<int>(kStageBytes);
   static constexpr size_t kSmem = static_cast<size_t>(kStages) * kStageBytes + kSmemReserve;
   // Tensor-memory accumulators (G: 128 columns, z: NZ columns each) cycled over tiles:
@@ -333,10 +336,17 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
 
 // GENERIC: binary16 weights or the Conv1D layout, chosen at run time; the default
 // instantiation (bf16, nn.Linear rows) has both folded away.
+// Chunks per ring stage: two for the default variant with a narrow v operand.
+template <int NZ, bool GENERIC>
+struct GramBps {
+  static constexpr int value = (!GENERIC && NZ <= 32) ? 2 : 1;
+};
+
 template <int NZ, int DH, bool FUSED, bool GENERIC>
 __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(const __grid_constant__ GramArgs a) {
   constexpr int NE = 32 * GramWarps<FUSED>::kEpiWarps;  // epilogue threads
-  using Cfg = GramCfg<NZ>;
+  constexpr int BPS = GramBps<NZ, GENERIC>::value;
+  using Cfg = GramCfg<NZ, BPS>;
   constexpr int S = Cfg::kStages;
   constexpr uint32_t SB = Cfg::kStageBytes;
   extern __shared__ uint8_t smem_raw[];
@@ -393,19 +403,25 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
         const CUtensorMap* map = tr.is_k ? &a.maps_k[tr.layer] : &a.maps_q[tr.layer];
         const int row0 = tr.idx * 128;
         const int vrow0 = (tr.layer * s.tiles_k + tr.idx) * NZ;
-        for (int kc = 0; kc < s.nkc; ++kc) {
+        for (int kc = 0; kc < s.nkc; kc += BPS) {
           const uint32_t st = issued % S, ph = (issued / S) & 1u;
           if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1u, abort, a.status)) { ok = false; break; }
           const uint32_t sx = smem_u32(smem + st * SB);
           const uint32_t fb = smem_u32(&full[st]);
-          mbar_arrive_expect_tx(fb, tr.is_k ? SB : kTileBytes);
-          if (cols) {  // out-features contiguous: two 64-row halves of the tile, MN-major
-            tma_load_2d(sx, map, fb, row0, kc * 64, pol);
-            tma_load_2d(sx + kTileBytes / 2, map, fb, row0 + 64, kc * 64, pol);
-          } else {
-            tma_load_3d(sx, map, fb, kc * 64, 0, row0 / DH, pol);  // 128/d_h heads of d_h rows
+          const int nb = (BPS > 1 && kc + 1 >= s.nkc) ? 1 : BPS;  // a ragged last stage holds one chunk
+          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * (tr.is_k ? kTileBytes + Cfg::kVBytes : kTileBytes));
+#pragma unroll
+          for (int b = 0; b < BPS; ++b) {
+            if (b >= nb) break;
+            const uint32_t bx = sx + b * kTileBytes;
+            if (cols) {  // out-features contiguous: two 64-row halves of the tile, MN-major
+              tma_load_2d(bx, map, fb, row0, (kc + b) * 64, pol);
+              tma_load_2d(bx + kTileBytes / 2, map, fb, row0 + 64, (kc + b) * 64, pol);
+            } else {
+              tma_load_3d(bx, map, fb, (kc + b) * 64, 0, row0 / DH, pol);  // 128/d_h heads of d_h rows
+            }
+            if (tr.is_k) tma_load_2d(sx + BPS * kTileBytes + b * Cfg::kVBytes, a.map_v, fb, (kc + b) * 64, vrow0, pol);
           }
-          if (tr.is_k) tma_load_2d(sx + kTileBytes, a.map_v, fb, kc * 64, vrow0, pol);
           ++issued;
         }
       }
@@ -429,20 +445,26 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
         tc_fence_after();
         const uint32_t dG = tmem + acc * 128u;
         const uint32_t dZ = tmem + NA * 128u + acc * static_cast<uint32_t>(NZ);
-        for (int kc = 0; kc < s.nkc; ++kc) {
+        for (int kc = 0; kc < s.nkc; kc += BPS) {
           const uint32_t st = consumed % S, ph = (consumed / S) & 1u;
           if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sx = smem_u32(smem + st * SB);
-          // K-major: +32 B per K16 step; MN-major (two 64-row atoms 8 KB apart): +2048 B
-          const uint64_t ad = cols ? desc_mnmajor_sw128_2atoms(sx, kTileBytes / 2) : desc_kmajor_sw128(sx);
-          const uint64_t astep = cols ? 128u : 2u;
-          const uint64_t vd = desc_kmajor_sw128(sx + kTileBytes);
+          const int nb = (BPS > 1 && kc + 1 >= s.nkc) ? 1 : BPS;
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const uint32_t accum = (kc | k) != 0 ? 1u : 0u;
-            umma_bf16(dG, ad + astep * k, ad + astep * k, idG, accum);
-            if (tr.is_k) umma_bf16(dZ, ad + astep * k, vd + 2u * k, idZ, accum);
+          for (int b = 0; b < BPS; ++b) {
+            if (b >= nb) break;
+            const uint32_t bx = sx + b * kTileBytes;
+            // K-major: +32 B per K16 step; MN-major (two 64-row atoms 8 KB apart): +2048 B
+            const uint64_t ad = cols ? desc_mnmajor_sw128_2atoms(bx, kTileBytes / 2) : desc_kmajor_sw128(bx);
+            const uint64_t astep = cols ? 128u : 2u;
+            const uint64_t vd = desc_kmajor_sw128(sx + BPS * kTileBytes + b * Cfg::kVBytes);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const uint32_t accum = ((kc + b) | k) != 0 ? 1u : 0u;
+              umma_bf16(dG, ad + astep * k, ad + astep * k, idG, accum);
+              if (tr.is_k) umma_bf16(dZ, ad + astep * k, vd + 2u * k, idZ, accum);
+            }
           }
           umma_commit(smem_u32(&empty[st]));
           ++consumed;
@@ -627,7 +649,7 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
 
 template <int NZ, int DH, bool FUSED, bool GENERIC>
 cudaError_t launch_gram_cfg(const GramArgs& a, int num_sms, cudaStream_t st) {
-  using Cfg = GramCfg<NZ>;
+  using Cfg = GramCfg<NZ, GramBps<NZ, GENERIC>::value>;
   auto kern = gram_kernel<NZ, DH, FUSED, GENERIC>;
   static bool configured = false;
   if (!configured) {
@@ -668,12 +690,18 @@ cudaError_t launch_gram_nz(const GramArgs& a, int num_sms, bool fused, cudaStrea
 
 }  // namespace
 
+template <int NZ>
+size_t gram_smem_max() {
+  const size_t a = GramCfg<NZ, GramBps<NZ, false>::value>::kSmem, b = GramCfg<NZ, GramBps<NZ, true>::value>::kSmem;
+  return a > b ? a : b;
+}
+
 size_t gram_smem_bytes(int nz) {
   switch (nz) {
-    case 16: return GramCfg<16>::kSmem;
-    case 32: return GramCfg<32>::kSmem;
-    case 64: return GramCfg<64>::kSmem;
-    case 128: return GramCfg<128>::kSmem;
+    case 16: return gram_smem_max<16>();
+    case 32: return gram_smem_max<32>();
+    case 64: return gram_smem_max<64>();
+    case 128: return gram_smem_max<128>();
     default: return 0;
   }
 }
