@@ -171,6 +171,27 @@ __device__ __forceinline__ float halfwarp_transpose_reduce8(float (&v)[8], int l
   return v[0];
 }
 
+// Sum of the NW per-warp partials of one head (NW = 4 or 8, 16-byte aligned).
+template <int NW>
+__device__ __forceinline__ float red_sum(const float* r) {
+  const float4 a = *reinterpret_cast<const float4*>(r);
+  float t = (a.x + a.y) + (a.z + a.w);
+  if (NW == 8) {
+    const float4 b = *reinterpret_cast<const float4*>(r + 4);
+    t += (b.x + b.y) + (b.z + b.w);
+  }
+  return t;
+}
+
+// The 8 consecutive entries rb .. rb+7 (rb a multiple of 8) of a vector in the plane layout.
+template <int CPT>
+__device__ __forceinline__ void load_rows8(const float* v, int rb, float (&o)[8]) {
+  const float4 a = *reinterpret_cast<const float4*>(v + vec_off<CPT>(rb));
+  const float4 b = *reinterpret_cast<const float4*>(v + vec_off<CPT>(rb + 4));
+  o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
+  o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
+}
+
 // k power iterations for the head(s) of one query tile, in R^{d_h}, run by the 8
 // epilogue warps.  Block layout: inside a head, warp w owns rows 16w + 8*(lane/16) .. +8
 // and lane % 16 owns d_h/16 consecutive columns, for both G_Q (copied once out of the
@@ -180,7 +201,9 @@ __device__ __forceinline__ float halfwarp_transpose_reduce8(float (&v)[8], int l
 // With x = c z (c a known scalar, c = 1 for z0) one iteration of Algorithm 2 is
 //   t' = G_Q x,  S1 = x.t' = c^2 sigma^2,  y = t' / sqrt(S1),
 //   w  = G_K y,  S2 = y.w = ||v'||^2,       x <- w,  c <- sqrt(S2),
-// two barriers per iteration.
+// two barriers per iteration.  Each thread's share of a dot product is taken from its
+// 8 row partials before they are reduced (S1 = sum over threads of sum_i x_i part_i),
+// so the dot product's warp sum runs beside the row reduction instead of after it.
 template <int DH>
 __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int idx, uint32_t tacc, int q,
                                               int half, int ew, int lane, EpiSmem* ep, volatile int* abort,
@@ -285,16 +308,18 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
       for (int k = 0; k < CPT; ++k) acc0 = fmaf(gq[i][k], xv[k], acc0);
       part[i] = acc0;
     }
+    float rv[8];
+    load_rows8<CPT>(xs, rb, rv);
+    float loc = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) loc = fmaf(rv[i], part[i], loc);
     const float tp = halfwarp_transpose_reduce8(part, lane, ridx);
+    float p = warp_sum(loc);
     const int row = rb + ridx;
-    const float xr = xs[vec_off<CPT>(row)];
     if (writer) ts[vec_off<CPT>(row)] = tp;
-    float p = warp_sum(writer ? xr * tp : 0.0f);
     if (lane == 0) ep->red[hs][0][ewh] = p;
     named_bar_sync(bar, NTH);
-    float s1 = 0.0f;
-#pragma unroll
-    for (int w = 0; w < NWH; ++w) s1 += ep->red[hs][0][w];
+    float s1 = red_sum<NWH>(ep->red[hs][0]);
     s1 = s1 < 0.0f ? 0.0f : s1;  // rounding can dip below 0; NaN must survive
     const float rs1 = sqrtf(s1);
     // zero guards that let a NaN through (x == 0 tests are false for NaN)
@@ -313,15 +338,18 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
       for (int k = 0; k < CPT; ++k) acc0 = fmaf(gk[i][k], xv[k], acc0);
       part[i] = acc0;
     }
+    // S2 = y.w = sum_i (t'_i / sqrt(S1)) (G_K t')_i / sqrt(S1)
+    load_rows8<CPT>(ts, rb, rv);
+    loc = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) loc = fmaf(rv[i] * inv1, part[i], loc);
     const float wrow = halfwarp_transpose_reduce8(part, lane, ridx) * inv1;
+    p = warp_sum(loc);
     y = tp * inv1;
     if (writer) xs[vec_off<CPT>(row)] = wrow;
-    p = warp_sum(writer ? y * wrow : 0.0f);
     if (lane == 0) ep->red[hs][1][ewh] = p;
     named_bar_sync(bar, NTH);
-    float s2 = 0.0f;
-#pragma unroll
-    for (int w = 0; w < NWH; ++w) s2 += ep->red[hs][1][w];
+    float s2 = red_sum<NWH>(ep->red[hs][1]) * inv1;
     s2 = s2 < 0.0f ? 0.0f : s2;
     n = sqrtf(s2);
     c = n;
