@@ -52,6 +52,8 @@ struct gas_ctx {
   float* ybuf = nullptr;
   CUtensorMap* dmaps = nullptr;  // [2L + 1]: q maps, k maps, v map
   unsigned* flags = nullptr;     // [L][tiles_k] key-tile flags of the fused kernel
+  unsigned* vflags = nullptr;    // [L][tiles_k] v-norm flags of the fused kernel
+  float* vn2 = nullptr;          // [L][nq] ||v||^2 of the start vectors (fused kernel)
   float* lz = nullptr;           // whole-layer path: z_kv [L][n_kv*d_h]
   float* lu = nullptr;           //                   u'   [L][d]
   float* ly = nullptr;           //                   y    [L][n_q*d_h]
@@ -113,6 +115,21 @@ bool encode_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, u
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// 2D fp32 map of the start vectors [rows][d] (row-major): box 64 columns x box_rows rows,
+// no swizzle (the fused Gram kernel's converter warps read the rows as loaded).
+bool encode_vrows(CUtensorMap* m, const void* base, uint64_t d, uint64_t rows, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {d, rows};
+  cuuint64_t strides[1] = {d * 4};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -294,16 +311,30 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
   gas_status gs = ensure_maps(h, wq, wk, st);
   if (gs != GAS_OK) return gs;
   int launches = 0;
-  gas::PrepArgs p{};
-  p.s = s;
-  p.v_in = v_in;
-  p.vhl = h->vhl;
-  p.s_zero = s_out;
-  p.epoch = h->epoch;
-  cudaError_t e = launch(h, "prep_v", st, [&] { return gas::launch_prep_v(p, st); });
+  cudaError_t e = cudaSuccess;
+  gas::GramArgs g{};
+  if (fused) {
+    // the fused kernel reads the fp32 v rows itself; a one-block prologue clears the
+    // per-layer scale slots and advances the flag epoch
+    if (!encode_vrows(&g.map_vf, v_in, static_cast<uint64_t>(s.d), static_cast<uint64_t>(s.L) * s.nq,
+                      static_cast<uint32_t>(s.nz / 2)))
+      return fail(h, GAS_ERR_CUDA, "cuTensorMapEncodeTiled failed for v_in");
+    gas::PrologueArgs p{};
+    p.L = s.L;
+    p.s_zero = s_out;
+    p.epoch = h->epoch;
+    e = launch(h, "prologue", st, [&] { return gas::launch_prologue(p, st); });
+  } else {
+    gas::PrepArgs p{};
+    p.s = s;
+    p.v_in = v_in;
+    p.vhl = h->vhl;
+    p.s_zero = s_out;
+    p.epoch = h->epoch;
+    e = launch(h, "prep_v", st, [&] { return gas::launch_prep_v(p, st); });
+  }
   ++launches;
   if (e == cudaSuccess) {
-    gas::GramArgs g{};
     g.s = s;
     g.maps_q = h->dmaps;
     g.maps_k = h->dmaps + s.L;
@@ -314,6 +345,8 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
     g.status = h->status;
     if (fused) {
       g.flags = h->flags;
+      g.vflags = h->vflags;
+      g.vn2 = h->vn2;
       g.epoch = h->epoch;
       g.iters = iters;
       g.ybuf = h->ybuf;
@@ -540,6 +573,8 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_y = take(L * NQ * DH * 4);
   const size_t o_maps = take((2 * L + 1) * sizeof(CUtensorMap));
   const size_t o_flags = take(L * s.tiles_k * sizeof(unsigned));
+  const size_t o_vflags = take(L * s.tiles_k * sizeof(unsigned));
+  const size_t o_vn2 = take(L * NQ * 4);
   const size_t o_lz = take(L * static_cast<size_t>(n_kv) * d_h * 4);
   const size_t o_lu = take(L * static_cast<size_t>(d) * 4);
   const size_t o_ly = take(L * static_cast<size_t>(n_q) * d_h * 4);
@@ -570,6 +605,8 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   h->ybuf = reinterpret_cast<float*>(b + o_y);
   h->dmaps = reinterpret_cast<CUtensorMap*>(b + o_maps);
   h->flags = reinterpret_cast<unsigned*>(b + o_flags);
+  h->vflags = reinterpret_cast<unsigned*>(b + o_vflags);
+  h->vn2 = reinterpret_cast<float*>(b + o_vn2);
   h->lz = reinterpret_cast<float*>(b + o_lz);
   h->lu = reinterpret_cast<float*>(b + o_lu);
   h->ly = reinterpret_cast<float*>(b + o_ly);

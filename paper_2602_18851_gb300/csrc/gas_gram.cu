@@ -9,12 +9,17 @@
 // iterations on 128 x 128 matrices (CUDA cores), and one more pass over B_g for the
 // write-back v_out = B^T y / ||v'||.
 //
-//   prep_v_kernel   v / ||v|| split into bf16 hi + lo rows (the tensor-core operand for z0)
+//   prep_v_kernel   (unfused) v / ||v|| split into bf16 hi + lo rows, the tensor-core
+//                   operand for z0
+//   prologue_kernel (fused) clears the per-layer scale slots, advances the flag epoch
 //   gram_kernel     persistent, warp-specialised: TMA -> smem ring -> tcgen05.mma into
 //                   TMEM; G = X X^T for every 128-row weight tile and, on key tiles,
-//                   Z = X [v_hi; v_lo]^T (z0 = B v in ~16-bit-mantissa precision)
-//   iterate_kernel  k iterations per head in R^{d_h} from G_Q, G_K, z0; sigma, y/||v'||,
-//                   fused per-layer scale (Eq. 15)
+//                   Z = X [v_hi; v_lo]^T (z0 = B v in ~16-bit-mantissa precision).  The
+//                   fused variant loads the fp32 v rows with the key tiles and splits
+//                   them into the hi / lo operand inside the ring (two converter warps),
+//                   which also sum ||v||^2 per head; its epilogue runs the k iterations
+//   iterate_kernel  (unfused) k iterations per head in R^{d_h} from G_Q, G_K, z0; sigma,
+//                   y/||v'||, fused per-layer scale (Eq. 15)
 // The write-back reuses the streaming K pass (gas_stream.cu).
 
 #include "gas_device.cuh"
@@ -23,24 +28,30 @@ namespace gas {
 
 namespace {
 
-// Warp 0: TMA producer; warp 1: MMA issuer (+ TMEM allocation); the rest: epilogue
-// (4 warps for the Gram-only kernel, 8 for the fused one: two threads per row).
+// Warp 0: TMA producer; warp 1: MMA issuer (+ TMEM allocation); then the epilogue
+// (4 warps for the Gram-only kernel, 8 for the fused one: two threads per row); the
+// fused kernel ends with 2 converter warps (fp32 v rows -> bf16 hi / lo MMA operand).
+// Twelve warps hold the same 168 registers per thread as ten (three warps per scheduler).
 template <bool FUSED>
 struct GramWarps {
   static constexpr int kEpiWarps = FUSED ? 8 : 4;
-  static constexpr int kThreads = 64 + 32 * kEpiWarps;
+  static constexpr int kConvWarps = FUSED ? 2 : 0;
+  static constexpr int kThreads = 64 + 32 * (kEpiWarps + kConvWarps);
 };
 constexpr uint32_t kTileBytes = 128u * 64u * 2u;  // one 128-row x 64-column bf16 box
 constexpr int kSmemBudget = 232448;               // 227 KB opt-in dynamic shared memory
 constexpr int kSmemReserve = 22528;               // alignment slack, barriers, epilogue scratch
 
-// A ring stage holds BPS consecutive 64-column chunks of a tile: BPS weight boxes, then
-// (key tiles) the BPS matching v boxes.  Two chunks per stage halve the per-byte count of
-// barrier waits, commits and copy issues on the producer and MMA threads.
-template <int NZ, int BPS>
+// A ring stage holds BPS consecutive 64-column chunks of a tile: BPS weight boxes, the
+// BPS matching v operand boxes (NZ rows of bf16 hi / lo, key tiles only) and, in the
+// fused kernel, the BPS fp32 v boxes they are converted from (NZ/2 rows x 64 floats).
+// Two chunks per stage halve the per-byte count of barrier waits, commits and copy
+// issues on the producer and MMA threads.
+template <int NZ, int BPS, bool FUSED>
 struct GramCfg {
   static constexpr uint32_t kVBytes = static_cast<uint32_t>(NZ) * 64u * 2u;
-  static constexpr uint32_t kStageBytes = BPS * (kTileBytes + kVBytes);
+  static constexpr uint32_t kFBytes = FUSED ? static_cast<uint32_t>(NZ / 2) * 64u * 4u : 0u;
+  static constexpr uint32_t kStageBytes = BPS * (kTileBytes + kVBytes + kFBytes);
   static constexpr int kStages = (kSmemBudget - kSmemReserve) / static_cast<int>(kStageBytes);
   static constexpr size_t kSmem = static_cast<size_t>(kStages) * kStageBytes + kSmemReserve;
   // Tensor-memory accumulators (G: 128 columns, z: NZ columns each) cycled over tiles:
@@ -92,6 +103,16 @@ __global__ void __launch_bounds__(256) prep_v_kernel(const __grid_constant__ Pre
   }
   if (a.s_zero != nullptr && h == 0 && threadIdx.x == 0) a.s_zero[l] = 0.0f;
   if (hidx == 0 && threadIdx.x == 0 && a.epoch != nullptr) {
+    const unsigned e = *a.epoch + 1u;
+    *a.epoch = e == 0u ? 1u : e;
+  }
+}
+
+// ---- fused path: per-layer scale slots cleared (atomic max target), flag epoch advanced --
+__global__ void __launch_bounds__(256) prologue_kernel(const __grid_constant__ PrologueArgs a) {
+  if (a.s_zero != nullptr)
+    for (int l = threadIdx.x; l < a.L; l += blockDim.x) a.s_zero[l] = 0.0f;
+  if (threadIdx.x == 0) {
     const unsigned e = *a.epoch + 1u;
     *a.epoch = e == 0u ? 1u : e;
   }
@@ -268,10 +289,13 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
   const int g = head / s.G;
   const int tk = (g * DH) / 128, og = (g * DH) % 128;
   const unsigned* flag = a.flags + layer * s.tiles_k + tk;
-  if (th == 0) ep->ok[hs] = wait_flag(flag, epoch, abort, a.status) ? 1 : 0;
+  const unsigned* vflag = a.vflags + layer * s.tiles_k + tk;
+  if (th == 0)
+    ep->ok[hs] = (wait_flag(flag, epoch, abort, a.status) && wait_flag(vflag, epoch, abort, a.status)) ? 1 : 0;
   named_bar_sync(bar, NTH);
   if (!ep->ok[hs]) return;
   (void)ld_acquire_u32(flag);
+  (void)ld_acquire_u32(vflag);
   // G_K is stored transposed: element (j, i) holds G_K[i][j]; rows rb.. are contiguous.
   const float* GK = a.gk + static_cast<size_t>(layer * s.tiles_k + tk) * 16384u + og * 128 + og;
   float gk[8][CPT];
@@ -286,8 +310,10 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
   // x and t' live in the plane layout (row stride 0: one "row" per slot).
   float* xs = &ep->xs[hs][0][0];
   float* ts = &ep->ts[hs][0][0];
-  if (th < DH)
-    xs[vec_off<CPT>(th)] = __ldcg(a.z0 + (hidx * 2) * DH + th) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + th);
+  if (th < DH) {  // z0 = B v from the unnormalised v rows: x = z0 / ||v|| (0 for a zero v)
+    const float inv = safe_inv_sqrt(__ldcg(a.vn2 + hidx));
+    xs[vec_off<CPT>(th)] = (__ldcg(a.z0 + (hidx * 2) * DH + th) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + th)) * inv;
+  }
   named_bar_sync(bar, NTH);
   const bool writer = (lane & 1) == 0;            // one of the two lanes holding a row total
   float c = 1.0f, sigma = 0.0f, y = 0.0f, n = 0.0f;
@@ -362,19 +388,21 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
   }
 }
 
-// GENERIC: binary16 weights or the Conv1D layout, chosen at run time; the default
-// instantiation (bf16, nn.Linear rows) has both folded away.
-// Chunks per ring stage: two for the default variant with a narrow v operand.
+// Chunks per ring stage: two when the v operand is narrow (at most 32 rows).
 template <int NZ, bool GENERIC>
 struct GramBps {
-  static constexpr int value = (!GENERIC && NZ <= 32) ? 2 : 1;
+  static constexpr int value = NZ <= 32 ? 2 : 1;
 };
 
+// GENERIC: binary16 weights or the Conv1D layout, chosen at run time; the default
+// instantiation (bf16, nn.Linear rows) has both folded away.
 template <int NZ, int DH, bool FUSED, bool GENERIC>
 __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(const __grid_constant__ GramArgs a) {
   constexpr int NE = 32 * GramWarps<FUSED>::kEpiWarps;  // epilogue threads
   constexpr int BPS = GramBps<NZ, GENERIC>::value;
-  using Cfg = GramCfg<NZ, BPS>;
+  using Cfg = GramCfg<NZ, BPS, FUSED>;
+  constexpr uint32_t kVOff = BPS * kTileBytes;                   // stage offset of the v operand boxes
+  constexpr uint32_t kFOff = BPS * (kTileBytes + Cfg::kVBytes);  // ... of the fp32 v boxes (fused)
   constexpr int S = Cfg::kStages;
   constexpr uint32_t SB = Cfg::kStageBytes;
   extern __shared__ uint8_t smem_raw[];
@@ -384,13 +412,15 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * SB);
   uint64_t* full = bars;
   uint64_t* empty = bars + S;
+  uint64_t* conv = bars + 2 * S;  // fused: the stage's v operand is converted
   constexpr int NA = Cfg::kAcc;
-  uint64_t* accf = bars + 2 * S;
+  uint64_t* accf = bars + 3 * S;
   uint64_t* acce = accf + NA;
   uint64_t* done = acce + NA;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  EpiSmem* ep = reinterpret_cast<EpiSmem*>(reinterpret_cast<uint8_t*>(done) + 64);
+  const uint32_t ep_off = ((smem_u32(done) + 64u + 127u) & ~127u) - smem_u32(smem);
+  EpiSmem* ep = reinterpret_cast<EpiSmem*>(smem + ep_off);
   volatile int no_abort_flag = 0;
 
   const Shape& s = a.s;
@@ -401,6 +431,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     for (int i = 0; i < S; ++i) {
       mbar_init(smem_u32(&full[i]), 1);
       mbar_init(smem_u32(&empty[i]), 1);
+      mbar_init(smem_u32(&conv[i]), 32 * GramWarps<FUSED>::kConvWarps + (FUSED ? 0 : 1));
     }
     for (int i = 0; i < NA; ++i) {
       mbar_init(smem_u32(&accf[i]), 1);
@@ -409,6 +440,13 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     mbar_init(smem_u32(done), 1);
     *abort = 0;
     fence_mbar_init();
+  }
+  if (FUSED) {
+    // v operand rows that no head uses (padding of NZ) must read as zero in every stage
+    for (int st = 0; st < S; ++st)
+      for (uint32_t o = threadIdx.x * 16u; o < BPS * Cfg::kVBytes; o += blockDim.x * 16u)
+        *reinterpret_cast<uint4*>(smem + st * SB + kVOff + o) = make_uint4(0, 0, 0, 0);
+    fence_proxy_async_smem();
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), 512);
@@ -437,7 +475,8 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           const uint32_t sx = smem_u32(smem + st * SB);
           const uint32_t fb = smem_u32(&full[st]);
           const int nb = (BPS > 1 && kc + 1 >= s.nkc) ? 1 : BPS;  // a ragged last stage holds one chunk
-          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * (tr.is_k ? kTileBytes + Cfg::kVBytes : kTileBytes));
+          const uint32_t vb = FUSED ? Cfg::kFBytes : Cfg::kVBytes;
+          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * (tr.is_k ? kTileBytes + vb : kTileBytes));
 #pragma unroll
           for (int b = 0; b < BPS; ++b) {
             if (b >= nb) break;
@@ -448,7 +487,13 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
             } else {
               tma_load_3d(bx, map, fb, (kc + b) * 64, 0, row0 / DH, pol);  // 128/d_h heads of d_h rows
             }
-            if (tr.is_k) tma_load_2d(sx + BPS * kTileBytes + b * Cfg::kVBytes, a.map_v, fb, (kc + b) * 64, vrow0, pol);
+            if (tr.is_k) {
+              if (FUSED)  // fp32 rows of the tile's heads: layer * nq + first head of the tile
+                tma_load_2d(sx + kFOff + b * Cfg::kFBytes, &a.map_vf, fb, (kc + b) * 64,
+                            tr.layer * s.nq + tr.idx * (128 / DH) * s.G, pol);
+              else
+                tma_load_2d(sx + kVOff + b * Cfg::kVBytes, a.map_v, fb, (kc + b) * 64, vrow0, pol);
+            }
           }
           ++issued;
         }
@@ -476,6 +521,9 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
         for (int kc = 0; kc < s.nkc; kc += BPS) {
           const uint32_t st = consumed % S, ph = (consumed / S) & 1u;
           if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
+          // Key tiles form a prefix of every CTA's tile list, so the converters' arrivals
+          // on conv[] follow the same stage sequence as full[] and share its parity.
+          if (FUSED && tr.is_k && !mbar_wait(smem_u32(&conv[st]), ph, abort, a.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sx = smem_u32(smem + st * SB);
           const int nb = (BPS > 1 && kc + 1 >= s.nkc) ? 1 : BPS;
@@ -486,7 +534,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
             // K-major: +32 B per K16 step; MN-major (two 64-row atoms 8 KB apart): +2048 B
             const uint64_t ad = cols ? desc_mnmajor_sw128_2atoms(bx, kTileBytes / 2) : desc_kmajor_sw128(bx);
             const uint64_t astep = cols ? 128u : 2u;
-            const uint64_t vd = desc_kmajor_sw128(sx + BPS * kTileBytes + b * Cfg::kVBytes);
+            const uint64_t vd = desc_kmajor_sw128(sx + kVOff + b * Cfg::kVBytes);
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               const uint32_t accum = ((kc + b) | k) != 0 ? 1u : 0u;
@@ -505,7 +553,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       umma_commit(smem_u32(done));
       mbar_wait(smem_u32(done), 0u, &no_abort_flag, a.status);
     }
-  } else {
+  } else if (warp < 2 + GramWarps<FUSED>::kEpiWarps) {
     // ---------------- epilogue: TMEM -> global ----------------
     const int q = warp & 3;  // tcgen05.ld: warp w may read TMEM lanes 32*(w%4) .. +31
     const int row = q * 32 + lane;
@@ -569,6 +617,82 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       tc_fence_before();
       mbar_arrive(smem_u32(&acce[acc]));
       ++tc;
+    }
+  } else if constexpr (FUSED) {
+    // ---------------- converters: fp32 v rows -> bf16 / f16 hi + lo operand rows --------
+    // Per key stage and chunk, thread ct takes 8 consecutive columns (one 16-byte unit of
+    // the SW128 K-major operand) of head row r = u / 8 for u = ct, ct + 64, ...; it writes
+    // the hi part to operand row gi*2G + j and the lo part to gi*2G + G + j (head j of
+    // group gi of the tile) and sums the squares of its v entries.  The rows are not
+    // normalised: the epilogue scales z0 by 1/||v|| from these sums.
+    constexpr int NC = 32 * GramWarps<FUSED>::kConvWarps;
+    constexpr int UMAX = (NZ / 2) * 8 / NC > 0 ? (NZ / 2) * 8 / NC : 1;
+    const int ct = threadIdx.x - 32 * (2 + GramWarps<FUSED>::kEpiWarps);
+    const int rt = (128 / DH) * s.G;  // head rows of a key tile (<= NZ / 2)
+    const unsigned epoch = __ldcg(a.epoch);
+    uint32_t cnt = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
+      const TileRef tr = decode_tile(s, t);
+      if (!tr.is_k) break;  // key tiles form a prefix of every CTA's tile list
+      float n2[UMAX];
+#pragma unroll
+      for (int i = 0; i < UMAX; ++i) n2[i] = 0.0f;
+      for (int kc = 0; kc < s.nkc; kc += BPS) {
+        const uint32_t st = cnt % S, ph = (cnt / S) & 1u;
+        if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
+        const int nb = (BPS > 1 && kc + 1 >= s.nkc) ? 1 : BPS;
+#pragma unroll
+        for (int b = 0; b < BPS; ++b) {
+          if (b >= nb) break;
+          const uint8_t* F = smem + st * SB + kFOff + b * Cfg::kFBytes;
+          uint8_t* V = smem + st * SB + kVOff + b * Cfg::kVBytes;
+#pragma unroll
+          for (int i = 0; i < UMAX; ++i) {
+            const int u = ct + NC * i;
+            const int r = u >> 3, c8 = u & 7;
+            if (r < rt) {
+              const float4 x0 = *reinterpret_cast<const float4*>(F + r * 256 + c8 * 32);
+              const float4 x1 = *reinterpret_cast<const float4*>(F + r * 256 + c8 * 32 + 16);
+              const float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+              uint32_t hb[8], lb[8];
+#pragma unroll
+              for (int e = 0; e < 8; ++e) {
+                n2[i] = fmaf(xv[e], xv[e], n2[i]);
+                split_hilo(xv[e], f16, hb[e], lb[e]);
+              }
+              const int gi = r / s.G, j = r - gi * s.G;
+              const int rh = gi * 2 * s.G + j, rl = rh + s.G;
+              *reinterpret_cast<uint4*>(V + rh * 128 + ((c8 ^ (rh & 7)) << 4)) =
+                  make_uint4(hb[0] | (hb[1] << 16), hb[2] | (hb[3] << 16), hb[4] | (hb[5] << 16), hb[6] | (hb[7] << 16));
+              *reinterpret_cast<uint4*>(V + rl * 128 + ((c8 ^ (rl & 7)) << 4)) =
+                  make_uint4(lb[0] | (lb[1] << 16), lb[2] | (lb[3] << 16), lb[4] | (lb[5] << 16), lb[6] | (lb[7] << 16));
+            }
+          }
+        }
+        fence_proxy_async_smem();  // the tensor core reads what these generic stores wrote
+        mbar_arrive(smem_u32(&conv[st]));
+        ++cnt;
+      }
+      if (!ok) break;
+      // ||v||^2 of every head of the tile, then this tile's v-norm flag
+      const int head0 = tr.idx * (128 / DH) * s.G;
+#pragma unroll
+      for (int i = 0; i < UMAX; ++i) {
+        float v2 = n2[i];
+        v2 += __shfl_xor_sync(0xFFFFFFFFu, v2, 1);
+        v2 += __shfl_xor_sync(0xFFFFFFFFu, v2, 2);
+        v2 += __shfl_xor_sync(0xFFFFFFFFu, v2, 4);
+        const int u = ct + NC * i;
+        const int r = u >> 3;
+        if ((u & 7) == 0 && r < rt && head0 + r < s.nq)
+          a.vn2[static_cast<size_t>(tr.layer) * s.nq + head0 + r] = v2;
+      }
+      named_bar_sync(6, NC);
+      if (ct == 0) {
+        __threadfence();
+        st_release_u32(a.vflags + tr.layer * s.tiles_k + tr.idx, epoch);
+      }
     }
   }
   tc_fence_before();
@@ -677,7 +801,7 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
 
 template <int NZ, int DH, bool FUSED, bool GENERIC>
 cudaError_t launch_gram_cfg(const GramArgs& a, int num_sms, cudaStream_t st) {
-  using Cfg = GramCfg<NZ, GramBps<NZ, GENERIC>::value>;
+  using Cfg = GramCfg<NZ, GramBps<NZ, GENERIC>::value, FUSED>;
   auto kern = gram_kernel<NZ, DH, FUSED, GENERIC>;
   static bool configured = false;
   if (!configured) {
@@ -720,8 +844,12 @@ cudaError_t launch_gram_nz(const GramArgs& a, int num_sms, bool fused, cudaStrea
 
 template <int NZ>
 size_t gram_smem_max() {
-  const size_t a = GramCfg<NZ, GramBps<NZ, false>::value>::kSmem, b = GramCfg<NZ, GramBps<NZ, true>::value>::kSmem;
-  return a > b ? a : b;
+  const size_t a = GramCfg<NZ, GramBps<NZ, false>::value, false>::kSmem;
+  const size_t b = GramCfg<NZ, GramBps<NZ, false>::value, true>::kSmem;
+  const size_t c = GramCfg<NZ, GramBps<NZ, true>::value, false>::kSmem;
+  const size_t d = GramCfg<NZ, GramBps<NZ, true>::value, true>::kSmem;
+  const size_t ab = a > b ? a : b, cd = c > d ? c : d;
+  return ab > cd ? ab : cd;
 }
 
 size_t gram_smem_bytes(int nz) {
@@ -736,6 +864,11 @@ size_t gram_smem_bytes(int nz) {
 
 cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st) {
   prep_v_kernel<<<a.s.L * a.s.nq, 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prologue(const PrologueArgs& a, cudaStream_t st) {
+  prologue_kernel<<<1, 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 

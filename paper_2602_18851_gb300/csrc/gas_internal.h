@@ -95,19 +95,31 @@ struct PrepArgs {
   unsigned* epoch;     // flag value of the next fused Gram launch (advanced here)
 };
 
+struct PrologueArgs {
+  int L;
+  float* s_zero;       // [L] or null
+  unsigned* epoch;     // flag value of the next fused Gram launch (advanced here)
+};
+
 struct GramArgs {
   Shape s;
+  // fused variant: fp32 v rows [L*nq][d], box 64 columns x nz/2 rows, no swizzle; a
+  // kernel parameter (re-encoded on the host for every call, no device upload)
+  CUtensorMap map_vf;
   const CUtensorMap* maps_q;  // [L] tensor maps over Wq[l] ([nq*dh, d], box 64 x 128)
   const CUtensorMap* maps_k;  // [L]
-  const CUtensorMap* map_v;   // one map over vhl ([L*tiles_k*nz, d], box 64 x nz)
+  const CUtensorMap* map_v;   // unfused: one map over vhl ([L*tiles_k*nz, d], box 64 x nz)
   float* gq;                  // [L][tiles_q][128][128] (unfused only)
   float* gk;                  // [L][tiles_k][128][128]
-  float* z0;                  // [L][nq][2][dh] (hi and lo halves of B_g v/||v||)
+  float* z0;                  // [L][nq][2][dh] hi and lo halves of B_g v/||v|| (unfused)
+                              // or of B_g v (fused)
   unsigned* status;
   // fused variant: k iterations in the epilogue, straight from tensor memory
   unsigned* flags;            // [L][tiles_k] key-tile publication flags (== epoch when ready)
   const unsigned* epoch;      // this launch's flag value (never 0), advanced on the device by
                               // prep_v_kernel, so that a replayed CUDA graph gets a new one
+  float* vn2;                 // [L][nq] ||v||^2 summed by the converter warps
+  unsigned* vflags;           // [L][tiles_k] v-norm flags (== epoch when vn2 of the tile is ready)
   int iters;
   float* ybuf;                // [L][nq][dh]
   float* sigma;               // [L][nq]
@@ -165,6 +177,7 @@ cudaError_t launch_stream_pass(const LayerTable& tab, const StreamArgs& a, cudaS
 cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st);
 cudaError_t launch_scales(const ScalesArgs& a, cudaStream_t st);
 cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st);
+cudaError_t launch_prologue(const PrologueArgs& a, cudaStream_t st);
 cudaError_t launch_gram(const GramArgs& a, int num_sms, bool fused, cudaStream_t st);
 cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st);
 cudaError_t launch_writeback(const WbArgs& a, int num_sms, cudaStream_t st);
