@@ -54,6 +54,9 @@ struct gas_ctx {
   unsigned* flags = nullptr;     // [L][tiles_k] key-tile flags of the fused kernel
   unsigned* vflags = nullptr;    // [L][tiles_k] v-norm flags of the fused kernel
   float* vn2 = nullptr;          // [L][nq] ||v||^2 of the start vectors (fused kernel)
+  unsigned* layer_cnt = nullptr;  // [L] finished heads per layer of the fused kernel
+  unsigned* done_cnt = nullptr;   // finished CTAs of the fused kernel
+  unsigned long long* layer_max = nullptr;  // [L] epoch-tagged sigma maxima of the fused kernel
   float* lz = nullptr;           // whole-layer path: z_kv [L][n_kv*d_h]
   float* lu = nullptr;           //                   u'   [L][d]
   float* ly = nullptr;           //                   y    [L][n_q*d_h]
@@ -314,16 +317,11 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
   cudaError_t e = cudaSuccess;
   gas::GramArgs g{};
   if (fused) {
-    // the fused kernel reads the fp32 v rows itself; a one-block prologue clears the
-    // per-layer scale slots and advances the flag epoch
+    // the fused kernel reads the fp32 v rows itself, writes the per-layer scales without a
+    // cleared accumulator and advances its flag epoch: it is the first launch of the call
     if (!encode_vrows(&g.map_vf, v_in, static_cast<uint64_t>(s.d), static_cast<uint64_t>(s.L) * s.nq,
                       static_cast<uint32_t>(s.nz / 2)))
       return fail(h, GAS_ERR_CUDA, "cuTensorMapEncodeTiled failed for v_in");
-    gas::PrologueArgs p{};
-    p.L = s.L;
-    p.s_zero = s_out;
-    p.epoch = h->epoch;
-    e = launch(h, "prologue", st, [&] { return gas::launch_prologue(p, st); });
   } else {
     gas::PrepArgs p{};
     p.s = s;
@@ -332,8 +330,8 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
     p.s_zero = s_out;
     p.epoch = h->epoch;
     e = launch(h, "prep_v", st, [&] { return gas::launch_prep_v(p, st); });
+    ++launches;
   }
-  ++launches;
   if (e == cudaSuccess) {
     g.s = s;
     g.maps_q = h->dmaps;
@@ -348,6 +346,9 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
       g.vflags = h->vflags;
       g.vn2 = h->vn2;
       g.epoch = h->epoch;
+      g.layer_cnt = h->layer_cnt;
+      g.layer_max = h->layer_max;
+      g.done_cnt = h->done_cnt;
       g.iters = iters;
       g.ybuf = h->ybuf;
       g.sigma = sigma;
@@ -575,6 +576,8 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_flags = take(L * s.tiles_k * sizeof(unsigned));
   const size_t o_vflags = take(L * s.tiles_k * sizeof(unsigned));
   const size_t o_vn2 = take(L * NQ * 4);
+  const size_t o_lcnt = take((L + 1) * sizeof(unsigned));
+  const size_t o_lmax = take(L * sizeof(unsigned long long));
   const size_t o_lz = take(L * static_cast<size_t>(n_kv) * d_h * 4);
   const size_t o_lu = take(L * static_cast<size_t>(d) * 4);
   const size_t o_ly = take(L * static_cast<size_t>(n_q) * d_h * 4);
@@ -589,6 +592,10 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   char* b = static_cast<char*>(h->ws);
   h->status = reinterpret_cast<unsigned*>(b + o_status);
   h->epoch = reinterpret_cast<unsigned*>(b + o_status + 128);
+  if (e == cudaSuccess) {  // flag epochs start at 1: a cleared flag (0) never reads as published
+    const unsigned one = 1u;
+    e = cudaMemcpy(h->epoch, &one, sizeof(one), cudaMemcpyHostToDevice);
+  }
   h->zp = reinterpret_cast<float*>(b + o_zp);
   h->n2p = reinterpret_cast<float*>(b + o_n2p);
   h->tp = reinterpret_cast<float*>(b + o_tp);
@@ -607,6 +614,9 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   h->flags = reinterpret_cast<unsigned*>(b + o_flags);
   h->vflags = reinterpret_cast<unsigned*>(b + o_vflags);
   h->vn2 = reinterpret_cast<float*>(b + o_vn2);
+  h->layer_cnt = reinterpret_cast<unsigned*>(b + o_lcnt);
+  h->done_cnt = h->layer_cnt + L;
+  h->layer_max = reinterpret_cast<unsigned long long*>(b + o_lmax);
   h->lz = reinterpret_cast<float*>(b + o_lz);
   h->lu = reinterpret_cast<float*>(b + o_lu);
   h->ly = reinterpret_cast<float*>(b + o_ly);

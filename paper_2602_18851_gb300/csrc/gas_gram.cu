@@ -11,7 +11,6 @@
 //
 //   prep_v_kernel   (unfused) v / ||v|| split into bf16 hi + lo rows, the tensor-core
 //                   operand for z0
-//   prologue_kernel (fused) clears the per-layer scale slots, advances the flag epoch
 //   gram_kernel     persistent, warp-specialised: TMA -> smem ring -> tcgen05.mma into
 //                   TMEM; G = X X^T for every 128-row weight tile and, on key tiles,
 //                   Z = X [v_hi; v_lo]^T (z0 = B v in ~16-bit-mantissa precision).  The
@@ -103,16 +102,6 @@ __global__ void __launch_bounds__(256) prep_v_kernel(const __grid_constant__ Pre
   }
   if (a.s_zero != nullptr && h == 0 && threadIdx.x == 0) a.s_zero[l] = 0.0f;
   if (hidx == 0 && threadIdx.x == 0 && a.epoch != nullptr) {
-    const unsigned e = *a.epoch + 1u;
-    *a.epoch = e == 0u ? 1u : e;
-  }
-}
-
-// ---- fused path: per-layer scale slots cleared (atomic max target), flag epoch advanced --
-__global__ void __launch_bounds__(256) prologue_kernel(const __grid_constant__ PrologueArgs a) {
-  if (a.s_zero != nullptr)
-    for (int l = threadIdx.x; l < a.L; l += blockDim.x) a.s_zero[l] = 0.0f;
-  if (threadIdx.x == 0) {
     const unsigned e = *a.epoch + 1u;
     *a.epoch = e == 0u ? 1u : e;
   }
@@ -384,7 +373,20 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
   if (th == 0) {
     a.sigma[hidx] = sigma;
     if (!isfinite(sigma)) set_status(a.status, GAS_DEV_NONFINITE_SIGMA);
-    if (a.scale_out != nullptr) atomic_max_nonneg(&a.scale_out[layer], a.scale_c * sigma);
+    if (a.scale_out != nullptr) {
+      // s_l = c * max_h sigma_{l,h} (Eq. 15): every head folds its sigma into an
+      // epoch-tagged maximum (epoch << 32 | bits; a word left by an earlier launch always
+      // loses, and on the bit patterns of non-negative floats a NaN wins), then the
+      // layer's last head writes the scale
+      const float w = sigma == 0.0f ? 0.0f : sigma;  // no -0.0
+      atomicMax(a.layer_max + layer, (static_cast<unsigned long long>(epoch) << 32) | __float_as_uint(w));
+      __threadfence();
+      if (atomicAdd(a.layer_cnt + layer, 1u) == static_cast<unsigned>(s.nq) - 1u) {
+        __threadfence();
+        const unsigned long long m = __ldcg(a.layer_max + layer);
+        a.scale_out[layer] = a.scale_c * __uint_as_float(static_cast<unsigned>(m));
+      }
+    }
   }
 }
 
@@ -474,7 +476,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1u, abort, a.status)) { ok = false; break; }
           const uint32_t sx = smem_u32(smem + st * SB);
           const uint32_t fb = smem_u32(&full[st]);
-          const int nb = (BPS > 1 && kc + 1 >= s.nkc) ? 1 : BPS;  // a ragged last stage holds one chunk
+          const int nb = min(BPS, s.nkc - kc);  // a ragged last stage holds fewer chunks
           const uint32_t vb = FUSED ? Cfg::kFBytes : Cfg::kVBytes;
           mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * (tr.is_k ? kTileBytes + vb : kTileBytes));
 #pragma unroll
@@ -526,7 +528,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           if (FUSED && tr.is_k && !mbar_wait(smem_u32(&conv[st]), ph, abort, a.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sx = smem_u32(smem + st * SB);
-          const int nb = (BPS > 1 && kc + 1 >= s.nkc) ? 1 : BPS;
+          const int nb = min(BPS, s.nkc - kc);
 #pragma unroll
           for (int b = 0; b < BPS; ++b) {
             if (b >= nb) break;
@@ -641,7 +643,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       for (int kc = 0; kc < s.nkc; kc += BPS) {
         const uint32_t st = cnt % S, ph = (cnt / S) & 1u;
         if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
-        const int nb = (BPS > 1 && kc + 1 >= s.nkc) ? 1 : BPS;
+        const int nb = min(BPS, s.nkc - kc);
 #pragma unroll
         for (int b = 0; b < BPS; ++b) {
           if (b >= nb) break;
@@ -701,6 +703,20 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, 512);
+  }
+  if (FUSED && threadIdx.x == 0) {
+    // The last CTA to finish (every CTA gets here, also after giving up on a bounded
+    // wait) clears the per-layer head counts and advances the flag epoch for the next
+    // launch; every CTA of this cooperative launch read the epoch at its start, and a
+    // replayed CUDA graph never takes this launch's flags for its own.
+    __threadfence();
+    if (atomicAdd(a.done_cnt, 1u) == gridDim.x - 1u) {
+      for (int l = 0; l < s.L; ++l) a.layer_cnt[l] = 0u;
+      *a.done_cnt = 0u;
+      const unsigned n = __ldcg(a.epoch) + 1u;
+      *a.epoch = n == 0u ? 1u : n;
+      __threadfence();
+    }
   }
 }
 
@@ -867,10 +883,7 @@ cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_prologue(const PrologueArgs& a, cudaStream_t st) {
-  prologue_kernel<<<1, 256, 0, st>>>(a);
-  return cudaGetLastError();
-}
+
 
 cudaError_t launch_gram(const GramArgs& a, int num_sms, bool fused, cudaStream_t st) {
   switch (a.s.nz) {

@@ -95,12 +95,6 @@ struct PrepArgs {
   unsigned* epoch;     // flag value of the next fused Gram launch (advanced here)
 };
 
-struct PrologueArgs {
-  int L;
-  float* s_zero;       // [L] or null
-  unsigned* epoch;     // flag value of the next fused Gram launch (advanced here)
-};
-
 struct GramArgs {
   Shape s;
   // fused variant: fp32 v rows [L*nq][d], box 64 columns x nz/2 rows, no swizzle; a
@@ -116,8 +110,11 @@ struct GramArgs {
   unsigned* status;
   // fused variant: k iterations in the epilogue, straight from tensor memory
   unsigned* flags;            // [L][tiles_k] key-tile publication flags (== epoch when ready)
-  const unsigned* epoch;      // this launch's flag value (never 0), advanced on the device by
-                              // prep_v_kernel, so that a replayed CUDA graph gets a new one
+  unsigned* epoch;            // this launch's flag value (never 0); the fused kernel's last CTA
+                              // advances it, so that a replayed CUDA graph gets a new one
+  unsigned* layer_cnt;        // [L] finished heads per layer (fused scales), cleared at the end
+  unsigned long long* layer_max;  // [L] epoch-tagged maximum sigma bits per layer
+  unsigned* done_cnt;         // finished CTAs
   float* vn2;                 // [L][nq] ||v||^2 summed by the converter warps
   unsigned* vflags;           // [L][tiles_k] v-norm flags (== epoch when vn2 of the tile is ready)
   int iters;
@@ -177,7 +174,6 @@ cudaError_t launch_stream_pass(const LayerTable& tab, const StreamArgs& a, cudaS
 cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st);
 cudaError_t launch_scales(const ScalesArgs& a, cudaStream_t st);
 cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st);
-cudaError_t launch_prologue(const PrologueArgs& a, cudaStream_t st);
 cudaError_t launch_gram(const GramArgs& a, int num_sms, bool fused, cudaStream_t st);
 cudaError_t launch_iterate(const IterArgs& a, cudaStream_t st);
 cudaError_t launch_writeback(const WbArgs& a, int num_sms, cudaStream_t st);
