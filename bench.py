@@ -163,7 +163,7 @@ def profiled_traffic(kernel, units):
     changed since the counters were taken."""
     import hashlib
     import re
-    files = {"gram_fused": ("gram_fused_llama2-70b-gqa-4layers.md", ["gas_gram.cu", "gas_device.cuh"]),
+    files = {"gram_fused": ("launches_llama2-70b-gqa.md", ["gas_gram.cu", "gas_device.cuh"]),
              "fp8_quantize": ("fp8_quantize_llama2-70b-layer-logits.md", ["gas_fp8.cu", "gas_device.cuh"])}
     if kernel not in files:
         return None
