@@ -112,19 +112,43 @@ struct TileRef {
   int layer, is_k, idx;
 };
 
-// Tile order: every key tile of every layer first, then the query tiles layer by layer,
-// so that a query tile's epilogue finds its key tile's G_K and z0 long published.
-__device__ __forceinline__ TileRef decode_tile(const Shape& s, int t) {
+// Tile order: the key tiles of the first D layers, then for every layer l the key tiles
+// of layer l + D (while there is such a layer) followed by the query tiles of layer l.
+// D layers of key tiles span at least two waves of the grid, so every query tile's key
+// tile comes at least two waves earlier in the order (and earlier in its own CTA's list):
+// its G_K and z0 are published in time, and every flag wait targets a smaller tile index,
+// so the waits form no cycle.  Between the first and last D layers key tiles, whose
+// epilogue is short, alternate with query tiles, whose epilogue runs the iterations: on
+// MHA shapes (as many key tiles as query tiles) this halves the epilogue's load there.
+// D = L puts every key tile first.
+__device__ __forceinline__ int lead_layers(const Shape& s, int grid) {
+  const int d = (2 * grid + s.tiles_k - 1) / s.tiles_k;
+  return d < s.L ? d : s.L;
+}
+
+__device__ __forceinline__ TileRef decode_tile(const Shape& s, int D, int t) {
   TileRef r;
-  const int nk = s.L * s.tiles_k;
-  r.is_k = t < nk;
-  if (r.is_k) {
-    r.layer = t / s.tiles_k;
-    r.idx = t - r.layer * s.tiles_k;
+  const int tk = s.tiles_k, tq = s.tiles_q;
+  const int P = D * tk;
+  if (t < P) {
+    r.is_k = 1;
+    r.layer = t / tk;
+    r.idx = t - r.layer * tk;
+    return r;
+  }
+  int u = t - P;
+  const int nf = s.L - D;  // layers whose block also carries the key tiles of layer l + D
+  const int fb = nf * (tk + tq);
+  if (u < fb) {
+    const int l = u / (tk + tq), q = u - l * (tk + tq);
+    r.is_k = q < tk;
+    r.layer = r.is_k ? l + D : l;
+    r.idx = r.is_k ? q : q - tk;
   } else {
-    const int u = t - nk;
-    r.layer = u / s.tiles_q;
-    r.idx = u - r.layer * s.tiles_q;
+    u -= fb;
+    r.is_k = 0;
+    r.layer = nf + u / tq;
+    r.idx = u - (r.layer - nf) * tq;
   }
   return r;
 }
@@ -414,9 +438,10 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * SB);
   uint64_t* full = bars;
   uint64_t* empty = bars + S;
-  uint64_t* conv = bars + 2 * S;  // fused: the stage's v operand is converted
+  uint64_t* conv = bars + 2 * S;   // fused key stages: the v operand is converted
+  uint64_t* vfull = bars + 3 * S;  // fused key stages: the fp32 v boxes have landed
   constexpr int NA = Cfg::kAcc;
-  uint64_t* accf = bars + 3 * S;
+  uint64_t* accf = bars + 4 * S;
   uint64_t* acce = accf + NA;
   uint64_t* done = acce + NA;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
@@ -434,6 +459,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       mbar_init(smem_u32(&full[i]), 1);
       mbar_init(smem_u32(&empty[i]), 1);
       mbar_init(smem_u32(&conv[i]), 32 * GramWarps<FUSED>::kConvWarps + (FUSED ? 0 : 1));
+      mbar_init(smem_u32(&vfull[i]), 1);
     }
     for (int i = 0; i < NA; ++i) {
       mbar_init(smem_u32(&accf[i]), 1);
@@ -459,15 +485,18 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int T = s.L * (s.tiles_k + s.tiles_q);
+  const int D = lead_layers(s, gridDim.x);
+  // Fused key stages: the conv[] and vfull[] barriers of stage st complete one phase per
+  // key-tile use of st; bit st of a role's kpar holds the parity of its next such phase.
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
     if (lane == 0) {
       const uint64_t pol = l2_policy_evict_first();
-      uint32_t issued = 0;
+      uint32_t issued = 0, kpar = 0u, kmask = 0u;  // kmask bit st: the latest use of st was a key stage
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
-        const TileRef tr = decode_tile(s, t);
+        const TileRef tr = decode_tile(s, D, t);
         const CUtensorMap* map = tr.is_k ? &a.maps_k[tr.layer] : &a.maps_q[tr.layer];
         const int row0 = tr.idx * 128;
         const int vrow0 = (tr.layer * s.tiles_k + tr.idx) * NZ;
@@ -477,8 +506,13 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           const uint32_t sx = smem_u32(smem + st * SB);
           const uint32_t fb = smem_u32(&full[st]);
           const int nb = min(BPS, s.nkc - kc);  // a ragged last stage holds fewer chunks
-          const uint32_t vb = FUSED ? Cfg::kFBytes : Cfg::kVBytes;
-          mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * (tr.is_k ? kTileBytes + vb : kTileBytes));
+          const uint32_t vfb = smem_u32(&vfull[st]);
+          if (FUSED) {
+            mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * kTileBytes);
+            if (tr.is_k) mbar_arrive_expect_tx(vfb, static_cast<uint32_t>(nb) * Cfg::kFBytes);
+          } else {
+            mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * (tr.is_k ? kTileBytes + Cfg::kVBytes : kTileBytes));
+          }
 #pragma unroll
           for (int b = 0; b < BPS; ++b) {
             if (b >= nb) break;
@@ -491,19 +525,28 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
             }
             if (tr.is_k) {
               if (FUSED)  // fp32 rows of the tile's heads: layer * nq + first head of the tile
-                tma_load_2d(sx + kFOff + b * Cfg::kFBytes, &a.map_vf, fb, (kc + b) * 64,
+                tma_load_2d(sx + kFOff + b * Cfg::kFBytes, &a.map_vf, vfb, (kc + b) * 64,
                             tr.layer * s.nq + tr.idx * (128 / DH) * s.G, pol);
               else
                 tma_load_2d(sx + kVOff + b * Cfg::kVBytes, a.map_v, fb, (kc + b) * 64, vrow0, pol);
             }
           }
+          if (FUSED) {
+            kmask = tr.is_k ? (kmask | (1u << st)) : (kmask & ~(1u << st));
+            if (tr.is_k) kpar ^= 1u << st;
+          }
           ++issued;
         }
       }
-      // Every copy still in flight targets this CTA's shared memory: wait for them to land.
+      // Every copy still in flight targets this CTA's shared memory: wait for them to land
+      // (the latest use of each stage; fp32 v boxes of key stages land on vfull[]).
       const uint32_t first = issued > static_cast<uint32_t>(S) ? issued - S : 0u;
-      for (uint32_t i = first; i < issued; ++i)
-        mbar_wait(smem_u32(&full[i % S]), (i / S) & 1u, &no_abort_flag, a.status);
+      for (uint32_t i = first; i < issued; ++i) {
+        const uint32_t st = i % S;
+        mbar_wait(smem_u32(&full[st]), (i / S) & 1u, &no_abort_flag, a.status);
+        if (FUSED && ((kmask >> st) & 1u))
+          mbar_wait(smem_u32(&vfull[st]), ((kpar >> st) & 1u) ^ 1u, &no_abort_flag, a.status);
+      }
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer (one thread) ----------------
@@ -511,10 +554,10 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       // Conv1D weights arrive MN-major (A and B of G = X X^T, A of Z = X V^T).
       const uint32_t idG = idesc_f32acc(128, 128, f16) | (cols ? (1u << 15) | (1u << 16) : 0u);
       const uint32_t idZ = idesc_f32acc(128, NZ, f16) | (cols ? (1u << 15) : 0u);
-      uint32_t consumed = 0, tc = 0;
+      uint32_t consumed = 0, tc = 0, kpar = 0u;
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
-        const TileRef tr = decode_tile(s, t);
+        const TileRef tr = decode_tile(s, D, t);
         const uint32_t acc = tc % NA, aph = (tc / NA) & 1u;
         if (!mbar_wait(smem_u32(&acce[acc]), aph ^ 1u, abort, a.status)) break;
         tc_fence_after();
@@ -523,9 +566,10 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
         for (int kc = 0; kc < s.nkc; kc += BPS) {
           const uint32_t st = consumed % S, ph = (consumed / S) & 1u;
           if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
-          // Key tiles form a prefix of every CTA's tile list, so the converters' arrivals
-          // on conv[] follow the same stage sequence as full[] and share its parity.
-          if (FUSED && tr.is_k && !mbar_wait(smem_u32(&conv[st]), ph, abort, a.status)) { ok = false; break; }
+          if (FUSED && tr.is_k) {
+            if (!mbar_wait(smem_u32(&conv[st]), (kpar >> st) & 1u, abort, a.status)) { ok = false; break; }
+            kpar ^= 1u << st;
+          }
           tc_fence_after();
           const uint32_t sx = smem_u32(smem + st * SB);
           const int nb = min(BPS, s.nkc - kc);
@@ -566,7 +610,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     const unsigned epoch = FUSED ? __ldcg(a.epoch) : 0u;
     uint32_t tc = 0;
     for (int t = blockIdx.x; t < T; t += gridDim.x) {
-      const TileRef tr = decode_tile(s, t);
+      const TileRef tr = decode_tile(s, D, t);
       const uint32_t acc = tc % NA, aph = (tc / NA) & 1u;
       const bool got = mbar_wait(smem_u32(&accf[acc]), aph, abort, a.status);
       __syncwarp();  // tcgen05.ld is warp-collective: reconverge after the per-lane wait
@@ -632,17 +676,21 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     const int ct = threadIdx.x - 32 * (2 + GramWarps<FUSED>::kEpiWarps);
     const int rt = (128 / DH) * s.G;  // head rows of a key tile (<= NZ / 2)
     const unsigned epoch = __ldcg(a.epoch);
-    uint32_t cnt = 0;
+    const uint32_t ns = static_cast<uint32_t>((s.nkc + BPS - 1) / BPS);  // stages per tile
+    uint32_t cnt = 0, kpar = 0u;
     bool ok = true;
     for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
-      const TileRef tr = decode_tile(s, t);
-      if (!tr.is_k) break;  // key tiles form a prefix of every CTA's tile list
+      const TileRef tr = decode_tile(s, D, t);
+      if (!tr.is_k) {  // query tiles: no v operand, only the stage count moves on
+        cnt += ns;
+        continue;
+      }
       float n2[UMAX];
 #pragma unroll
       for (int i = 0; i < UMAX; ++i) n2[i] = 0.0f;
       for (int kc = 0; kc < s.nkc; kc += BPS) {
-        const uint32_t st = cnt % S, ph = (cnt / S) & 1u;
-        if (!mbar_wait(smem_u32(&full[st]), ph, abort, a.status)) { ok = false; break; }
+        const uint32_t st = cnt % S;
+        if (!mbar_wait(smem_u32(&vfull[st]), (kpar >> st) & 1u, abort, a.status)) { ok = false; break; }
         const int nb = min(BPS, s.nkc - kc);
 #pragma unroll
         for (int b = 0; b < BPS; ++b) {
@@ -674,6 +722,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
         }
         fence_proxy_async_smem();  // the tensor core reads what these generic stores wrote
         mbar_arrive(smem_u32(&conv[st]));
+        kpar ^= 1u << st;
         ++cnt;
       }
       if (!ok) break;
