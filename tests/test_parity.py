@@ -193,6 +193,33 @@ def test_zero_start_vectors_and_inplace_warm_start(method):
 
 
 @pytest.mark.parametrize("method", METHODS)
+@pytest.mark.parametrize("name", ["tiny-gqa128", "ragged"])
+def test_start_vector_scale(name, method):
+    """Algorithm 2 starts from v / ||v||: sigma and v_out do not depend on the scale of
+    the start vectors.  Per-head scales from 2^-20 to 2^20 and non-powers of two, at
+    k = 1 (where the first sigma is ||M v|| / ||v||), 2 and the workload's count: the
+    library matches the oracle (which normalises first) and, to 1e-4, its own unscaled
+    run."""
+    wl = get_workload(name)
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    gen = torch.Generator().manual_seed(7)
+    exps = torch.randint(-20, 21, (wl.layers, wl.n_q), generator=gen).double()
+    scale = torch.pow(2.0, exps)
+    scale[0, 0], scale[-1, -1] = 3.7e-5, 1234.5
+    v_scaled = (v_in.double().cpu() * scale[..., None]).float().to(v_in.device)
+    for iters in (1, 2, wl.iters):
+        base = run_library(wl, wq, wk, v_in, method=method, iters=iters)
+        got = run_library(wl, wq, wk, v_scaled, method=method, iters=iters)
+        sig, v = oracle_for(wl, wq, wk, v_scaled, iters=iters)
+        assert_sigma_close(got["sigma"].ravel(), sig)
+        assert_v_close(got["v_out"], v)
+        # the 16-bit hi/lo operand of v rounds differently for non-power-of-two scales
+        assert_sigma_close(got["sigma"].ravel(), base["sigma"].ravel(), rtol=1e-4, what="sigma vs unscaled")
+        assert_v_close(got["v_out"], base["v_out"].reshape(-1, wl.d), atol=1e-4)
+        assert got["status"] == 0
+
+
+@pytest.mark.parametrize("method", METHODS)
 def test_nonfinite_weights_flag_status(method):
     import paper_2602_18851_gb300 as gas
     wl = get_workload("tiny-gqa")
