@@ -114,15 +114,15 @@ struct TileRef {
 
 // Tile order: the key tiles of the first D layers, then for every layer l the key tiles
 // of layer l + D (while there is such a layer) followed by the query tiles of layer l.
-// D layers of key tiles span at least two waves of the grid, so every query tile's key
-// tile comes at least two waves earlier in the order (and earlier in its own CTA's list):
-// its G_K and z0 are published in time, and every flag wait targets a smaller tile index,
-// so the waits form no cycle.  Between the first and last D layers key tiles, whose
-// epilogue is short, alternate with query tiles, whose epilogue runs the iterations: on
-// MHA shapes (as many key tiles as query tiles) this halves the epilogue's load there.
-// D = L puts every key tile first.
+// D layers of key tiles span at least one wave of the grid, so every query tile's key
+// tile comes at least one wave earlier in the order (and earlier in its own CTA's list):
+// its G_K and z0 are normally published by the time the query tile's epilogue starts,
+// and every flag wait targets a smaller tile index, so the waits form no cycle.  Between
+// the first and last D layers key tiles, whose epilogue is short, alternate with query
+// tiles, whose epilogue runs the iterations: on MHA shapes (as many key tiles as query
+// tiles) this halves the epilogue's load there.  D = L puts every key tile first.
 __device__ __forceinline__ int lead_layers(const Shape& s, int grid) {
-  const int d = (2 * grid + s.tiles_k - 1) / s.tiles_k;
+  const int d = (grid + s.tiles_k - 1) / s.tiles_k;
   return d < s.L ? d : s.L;
 }
 
