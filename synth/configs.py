@@ -75,6 +75,9 @@ WORKLOADS = {
     # widest z0 / write-back operand, 128 rows).
     "tiny-g16": Workload("tiny-g16", 2, 384, 16, 1, 128, 8, "spike4", _BASE_SEED + 16),
     "tiny-g32": Workload("tiny-g32", 2, 320, 32, 1, 64, 8, "spike4", _BASE_SEED + 17),
+    # The largest group at d_h 128: 64 query heads per KV head (a 128-row v operand and
+    # 64 heads' start vectors per key tile).
+    "tiny-g64": Workload("tiny-g64", 2, 256, 64, 1, 128, 6, "spike4", _BASE_SEED + 21),
     # Head widths outside {64, 128} (streaming back end): 80 and 96 as in several
     # published models, 256 as in wide-head ones.
     "tiny-dh80": Workload("tiny-dh80", 2, 320, 4, 2, 80, 10, "spike4", _BASE_SEED + 18),

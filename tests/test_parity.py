@@ -17,7 +17,7 @@ from tests.parity_utils import (assert_sigma_close, assert_v_close, gpu_inputs, 
 pytestmark = pytest.mark.gpu
 
 METHODS = ["fused", "gram", "stream"]
-SMALL = ["tiny-mha", "tiny-gqa", "tiny-gqa128", "ragged", "ragged128", "tiny-g16", "tiny-g32",
+SMALL = ["tiny-mha", "tiny-gqa", "tiny-gqa128", "ragged", "ragged128", "tiny-g16", "tiny-g32", "tiny-g64",
          "gpt2-small"]
 
 
