@@ -19,7 +19,7 @@
 //                   which also sum ||v||^2 per head; its epilogue runs the k iterations
 //   iterate_kernel  (unfused) k iterations per head in R^{d_h} from G_Q, G_K, z0; sigma,
 //                   y/||v'||, fused per-layer scale (Eq. 15)
-// The write-back reuses the streaming K pass (gas_stream.cu).
+// The write-back v_out = B^T y / ||v'|| is its own tensor-core kernel (gas_writeback.cu).
 
 #include "gas_device.cuh"
 
@@ -431,6 +431,8 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   constexpr uint32_t kFOff = BPS * (kTileBytes + Cfg::kVBytes);  // ... of the fp32 v boxes (fused)
   constexpr int S = Cfg::kStages;
   constexpr uint32_t SB = Cfg::kStageBytes;
+  static_assert(1023 + (4 * S + 2 * Cfg::kAcc + 1) * 8 + 64 + 127 + sizeof(EpiSmem) <= kSmemReserve,
+                "alignment slack, barriers and epilogue scratch must fit in the reserve");
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment by pointer arithmetic on the shared array itself, so that the
   // compiler keeps every derived pointer in the shared address space.
