@@ -20,30 +20,23 @@ namespace {
 
 constexpr int kRowBlock = 64;  // rows per rowdot CTA (8 warps x 8 rows)
 
-// Stage src[0..n) * (1/||src||) (or * 1 when normalise == 0) into shared memory.
-__device__ __forceinline__ void stage_vector(float* xs, const float* src, int n, int normalise, float* red) {
-  float n2 = 0.0f;
-  if (normalise) {
-    for (int i = threadIdx.x * 4; i < n; i += blockDim.x * 4) {
-      const float4 v = *reinterpret_cast<const float4*>(src + i);
-      n2 = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, n2))));
-    }
-    n2 = warp_sum(n2);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = n2;
-    __syncthreads();
-    n2 = 0.0f;
-    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) n2 += red[w];
-  }
-  const float inv = normalise ? safe_inv_sqrt(n2) : 1.0f;
-  for (int i = threadIdx.x * 4; i < n; i += blockDim.x * 4) {
-    float4 v = *reinterpret_cast<const float4*>(src + i);
-    v.x *= inv; v.y *= inv; v.z *= inv; v.w *= inv;
-    *reinterpret_cast<float4*>(xs + i) = v;
-  }
-  __syncthreads();
+// 8 weights of row r at column c (zero beyond the matrix) and their dot with x[c .. c+8).
+template <int WT>
+__device__ __forceinline__ float dot8(const W8<WT>& q, const float* xs, int c) {
+  const float4 x0 = *reinterpret_cast<const float4*>(xs + c);
+  const float4 x1 = *reinterpret_cast<const float4*>(xs + c + 4);
+  float f[8];
+  unpack_w8<WT>(q, f);
+  float t = f[0] * x0.x;
+  t = fmaf(f[1], x0.y, t); t = fmaf(f[2], x0.z, t); t = fmaf(f[3], x0.w, t);
+  t = fmaf(f[4], x1.x, t); t = fmaf(f[5], x1.y, t); t = fmaf(f[6], x1.z, t);
+  return fmaf(f[7], x1.w, t);
 }
 
-// out[l][r] = sum_c W_l[r][c] * x_l[c] for a block of 64 rows; x = src/||src|| (d values).
+// out[l][r] = sum_c W_l[r][c] * x_l[c] / ||x_l|| for a block of 64 rows (d values of x).
+// x is staged unnormalised while its squared norm is summed, and the 64 results are
+// scaled at the end.  Each lane keeps 16 weight loads in flight (8 rows x 2 column
+// blocks of 256).
 template <int WT>
 __global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant__ LayerTable tab,
                                                            const __grid_constant__ LayerArgs a) {
@@ -53,34 +46,54 @@ __global__ void __launch_bounds__(256) layer_rowdot_kernel(const __grid_constant
   const int l = blockIdx.y;
   const bool isq = a.which == 1;
   const int R = (isq ? a.s.nq : a.s.nkv) * a.s.dh;
+  const int d = a.s.d;
   const void* W = isq ? tab.q[l] : tab.k[l];
   const long long ld = isq ? a.s.ldq : a.s.ldk;
   const long long hstride = isq ? a.s.hsq : a.s.hsk;
-  stage_vector(xs, a.src + static_cast<size_t>(l) * a.s.d, a.s.d, 1, red);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  {
+    const float* src = a.src + static_cast<size_t>(l) * d;
+    float n2 = 0.0f;
+    for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
+      const float4 v = *reinterpret_cast<const float4*>(src + i);
+      n2 = fmaf(v.x, v.x, fmaf(v.y, v.y, fmaf(v.z, v.z, fmaf(v.w, v.w, n2))));
+      *reinterpret_cast<float4*>(xs + i) = v;
+    }
+    n2 = warp_sum(n2);
+    if (lane == 0) red[warp] = n2;
+    __syncthreads();
+  }
+  float n2 = 0.0f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) n2 += red[w];
+  const float inv = safe_inv_sqrt(n2);
   const int r0 = blockIdx.x * kRowBlock + warp * 8;
+  long long roff[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) roff[i] = weight_row_offset(r0 + i < R ? r0 + i : r0, a.s.dh, ld, hstride);
   float acc[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) acc[i] = 0.0f;
-  for (int c = lane * 8; c < a.s.d; c += 256) {
-    const float4 x0 = *reinterpret_cast<const float4*>(xs + c);
-    const float4 x1 = *reinterpret_cast<const float4*>(xs + c + 4);
-    const float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+  for (int c = lane * 8; c < d; c += 512) {
+    const int c2 = c + 256;
+    const bool two = c2 < d;
+    W8<WT> q0[8], q1[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      if (r0 + i < R) {
-        const W8<WT> q = load_w8<WT>(W, weight_row_offset(r0 + i, a.s.dh, ld, hstride) + c);
-        float f[8];
-        unpack_w8<WT>(q, f);
+      const bool ok = r0 + i < R;
+      q0[i] = ok ? load_w8<WT>(W, roff[i] + c) : zero_w8<WT>();
+      q1[i] = (ok && two) ? load_w8<WT>(W, roff[i] + c2) : zero_w8<WT>();
+    }
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[i] = fmaf(f[e], xv[e], acc[i]);
-      }
+    for (int i = 0; i < 8; ++i) {
+      acc[i] += dot8<WT>(q0[i], xs, c);
+      if (two) acc[i] += dot8<WT>(q1[i], xs, c2);
     }
   }
   int idx;
   const float tot = warp_transpose_reduce<8>(acc, lane, idx);
   if (transpose_reduce_writer<8>(lane) && r0 + idx < R)
-    a.out[static_cast<size_t>(l) * a.out_stride + r0 + idx] = tot;
+    a.out[static_cast<size_t>(l) * a.out_stride + r0 + idx] = tot * inv;
 }
 
 // out[l][c] = sum_r W_l[r][c] * x_l[r] for a chunk of 256 columns over all rows, with
@@ -118,8 +131,22 @@ __global__ void __launch_bounds__(256) layer_coldot_kernel(const __grid_constant
 #pragma unroll
   for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
   if (c < s.d) {
-#pragma unroll 4
-    for (int r = warp; r < R; r += 8) {
+    // warp w takes rows w, w + 8, ...; eight of them are loaded before any is used
+    int r = warp;
+    for (; r + 56 < R; r += 64) {
+      W8<WT> q[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) q[j] = load_w8<WT>(W, weight_row_offset(r + 8 * j, s.dh, ld, hstride) + c);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        float f[8];
+        unpack_w8<WT>(q[j], f);
+        const float xr = xs[r + 8 * j];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] = fmaf(f[e], xr, acc[e]);
+      }
+    }
+    for (; r < R; r += 8) {
       const W8<WT> q = load_w8<WT>(W, weight_row_offset(r, s.dh, ld, hstride) + c);
       float f[8];
       unpack_w8<WT>(q, f);
