@@ -73,10 +73,12 @@ typedef enum {
  * Create a handle for one model shape (the paper's Section 4 cost model
  * O(n_q * d_h * d) per layer per iteration).
  *   layers >= 1; d >= 8 and d % 8 == 0 (16-byte rows); n_q, n_kv >= 1 with
- *   n_q % n_kv == 0; d_h in {64, 80, 96, 128, 256}; for d_h 64 / 128 the group size
- *   n_q/n_kv <= 64 (d_h 128) or 32 (d_h 64).  The tensor-core back ends (fused, gram)
- *   need d_h 64 or 128 and 16-bit weights; other head widths and fp32 weights run on
- *   the streaming back end, which GAS_METHOD_AUTO then selects.
+ *   n_q % n_kv == 0; d_h in {64, 80, 96, 128, 256}; for d_h 64 / 80 / 96 / 128 the
+ *   group size n_q/n_kv <= 32 (d_h 64) or 64 (the others).  The tensor-core back ends
+ *   (fused, gram) need d_h 64, 80, 96 or 128 (a d_h 80 / 96 head fills the top rows of
+ *   a 128-row tile, the rest reads as zero), 16-bit weights, and for the Conv1D layout
+ *   d_h 64 or 128; d_h 256 and fp32 weights run on the streaming back end, which
+ *   GAS_METHOD_AUTO then selects.
  * Allocates the device workspace on the current device (see gas_workspace_bytes).
  * Errors: GAS_ERR_INVALID_ARG (out == NULL, non-positive sizes), GAS_ERR_UNSUPPORTED
  * (shape limits above), GAS_ERR_ALLOC, GAS_ERR_CUDA.  *out is NULL on error.

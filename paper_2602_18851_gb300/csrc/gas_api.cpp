@@ -138,15 +138,16 @@ bool encode_vrows(CUtensorMap* m, const void* base, uint64_t d, uint64_t rows, u
 }
 
 // 3D bf16 map of one weight matrix: (column c, row i inside a head, head j) at
-// base + j * hs + i * ld + c; box 64 columns x d_h rows x 128/d_h heads, so a box is one
-// 128-row tile in the canonical K-major SW128 layout whatever the strides.
+// base + j * hs + i * ld + c; box 64 columns x d_h rows x hpt heads (128 / tile head
+// width), so a box fills the top d_h * hpt rows of one 128-row tile in the canonical
+// K-major SW128 layout whatever the strides (all 128 rows unless d_h is 80 or 96).
 bool encode_weights(CUtensorMap* m, const void* base, uint64_t d, uint32_t dh, uint64_t heads, uint64_t ld,
-                    uint64_t hs) {
+                    uint64_t hs, uint32_t hpt) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[3] = {d, dh, heads};
   cuuint64_t strides[2] = {ld * 2, hs * 2};
-  cuuint32_t box[3] = {64, dh, 128 / dh};
+  cuuint32_t box[3] = {64, dh, hpt};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -196,8 +197,8 @@ gas_status ensure_maps(gas_ctx* h, const void* const* wq, const void* const* wk,
     const bool ok =
         sh.cols ? encode_cols(&h->hmaps[l], wq[l], static_cast<uint64_t>(sh.nq) * sh.dh, sh.d, sh.ldq) &&
                       encode_cols(&h->hmaps[L + l], wk[l], static_cast<uint64_t>(sh.nkv) * sh.dh, sh.d, sh.ldk)
-                : encode_weights(&h->hmaps[l], wq[l], sh.d, sh.dh, sh.nq, sh.ldq, sh.hsq) &&
-                      encode_weights(&h->hmaps[L + l], wk[l], sh.d, sh.dh, sh.nkv, sh.ldk, sh.hsk);
+                : encode_weights(&h->hmaps[l], wq[l], sh.d, sh.dh, sh.nq, sh.ldq, sh.hsq, sh.dh == 64 ? 2 : 1) &&
+                      encode_weights(&h->hmaps[L + l], wk[l], sh.d, sh.dh, sh.nkv, sh.ldk, sh.hsk, sh.dh == 64 ? 2 : 1);
     if (!ok)
       return fail(h, GAS_ERR_CUDA, "cuTensorMapEncodeTiled failed for layer %d", l);
     h->map_q[l] = wq[l];
@@ -310,7 +311,9 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
 gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, const gas::LayerTable& tab,
                     int iters, const float* v_in, float* v_out, float* sigma, float* s_out, float scale_c,
                     bool fused, cudaStream_t st) {
-  const Shape& s = h->s;
+  // the tensor-core kernels see the tile head width (rows past the model's d_h are zero)
+  Shape s = h->s;
+  s.dh = s.rows == 64 ? 64 : 128;
   gas_status gs = ensure_maps(h, wq, wk, st);
   if (gs != GAS_OK) return gs;
   int launches = 0;
@@ -405,11 +408,12 @@ gas_status spectral_impl(gas_ctx* h, const void* const* wq, const void* const* w
   gas::LayerTable tab;
   std::memset(&tab, 0, sizeof(tab));
   fill_table(h, tab, wq, wk);
-  const bool tc_ok = h->s.tc && !h->s.f32;
+  // Conv1D tiles are read as 64-row boxes of whole heads: d_h 64 or 128 only
+  const bool tc_ok = h->s.tc && !h->s.f32 && (!h->s.cols || h->s.dh == 64 || h->s.dh == 128);
   const int method = h->method == GAS_METHOD_AUTO ? (tc_ok ? GAS_METHOD_FUSED : GAS_METHOD_STREAM) : h->method;
   if (method != GAS_METHOD_STREAM && !tc_ok)
-    return fail(h, GAS_ERR_UNSUPPORTED, "the tensor-core back ends need d_h 64 or 128 and 16-bit weights "
-                                        "(use GAS_METHOD_STREAM or AUTO)");
+    return fail(h, GAS_ERR_UNSUPPORTED, "the tensor-core back ends need d_h 64, 80, 96 or 128, 16-bit weights, "
+                                        "and d_h 64 or 128 in the Conv1D layout (use GAS_METHOD_STREAM or AUTO)");
   if (method == GAS_METHOD_STREAM && h->s.f32 && h->s.dh > 128)
     return fail(h, GAS_ERR_UNSUPPORTED, "fp32 weights are supported up to d_h 128");
   if (method == GAS_METHOD_STREAM && h->s.cols)
@@ -509,10 +513,12 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   if (d_h != 64 && d_h != 80 && d_h != 96 && d_h != 128 && d_h != 256)
     return fail(nullptr, GAS_ERR_UNSUPPORTED, "d_h must be 64, 80, 96, 128 or 256 (got %d)", d_h);
   const int G = n_q / n_kv;
-  // d_h 64 / 128: whole heads fill 128-row tiles and the tensor-core back ends apply;
-  // other head widths run on the streaming back end only.
-  const bool tc = d_h == 64 || d_h == 128;
-  const int gpt = tc ? 128 / d_h : 1;
+  // d_h 64 / 128: whole heads fill 128-row tiles; d_h 80 / 96: one head per 128-row tile,
+  // the rows past d_h zero.  These run on the tensor-core back ends; d_h 256 runs on the
+  // streaming back end only.
+  const bool tc = d_h == 64 || d_h == 80 || d_h == 96 || d_h == 128;
+  const int dh_t = d_h == 64 ? 64 : 128;  // head width of a tensor-core tile
+  const int gpt = tc ? 128 / dh_t : 1;
   const int nz = round_up16(2 * G * gpt);
   if (tc && nz > 128)
     return fail(nullptr, GAS_ERR_UNSUPPORTED, "group size %d too large for d_h %d (max %d)", G, d_h, 64 / gpt);
@@ -523,8 +529,8 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   Shape& s = h->s;
   s.L = layers; s.d = d; s.nq = n_q; s.nkv = n_kv; s.dh = d_h; s.G = G;
   s.nch = (d + gas::kStreamChunk - 1) / gas::kStreamChunk;
-  s.tiles_q = (n_q * d_h + 127) / 128;
-  s.tiles_k = (n_kv * d_h + 127) / 128;
+  s.tiles_q = (n_q * dh_t + 127) / 128;
+  s.tiles_k = (n_kv * dh_t + 127) / 128;
   s.nkc = (d + 63) / 64;
   s.nz = nz_t;
   s.ldq = s.ldk = d;
@@ -533,6 +539,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   s.cols = 0;
   s.f32 = 0;
   s.tc = tc ? 1 : 0;
+  s.rows = d_h;
 
   cudaError_t e = cudaGetDevice(&h->device);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
@@ -570,8 +577,8 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_vhl = take(L * s.tiles_k * static_cast<size_t>(s.nz) * d * 2);
   const size_t o_gq = take(L * s.tiles_q * 16384ull * 4);
   const size_t o_gk = take(L * s.tiles_k * 16384ull * 4);
-  const size_t o_z0 = take(L * NQ * 2 * DH * 4);
-  const size_t o_y = take(L * NQ * DH * 4);
+  const size_t o_z0 = take(L * NQ * 2 * static_cast<size_t>(dh_t) * 4);
+  const size_t o_y = take(L * NQ * static_cast<size_t>(dh_t) * 4);
   const size_t o_maps = take((2 * L + 1) * sizeof(CUtensorMap));
   const size_t o_flags = take(L * s.tiles_k * sizeof(unsigned));
   const size_t o_vflags = take(L * s.tiles_k * sizeof(unsigned));

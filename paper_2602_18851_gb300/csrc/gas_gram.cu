@@ -471,13 +471,22 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     *abort = 0;
     fence_mbar_init();
   }
+  // Bytes one weight box brings: 128 rows, or d_h of them when a d_h 80 / 96 head sits in
+  // a 128-row tile; the rows below stay zero (written once here, never by TMA).
+  const uint32_t wbox = cols ? kTileBytes : static_cast<uint32_t>((128 / DH) * s.rows) * 128u;
+  if (wbox < kTileBytes) {
+    for (int st = 0; st < S; ++st)
+      for (int b = 0; b < BPS; ++b)
+        for (uint32_t o = wbox + threadIdx.x * 16u; o < kTileBytes; o += blockDim.x * 16u)
+          *reinterpret_cast<uint4*>(smem + st * SB + b * kTileBytes + o) = make_uint4(0, 0, 0, 0);
+  }
   if (FUSED) {
     // v operand rows that no head uses (padding of NZ) must read as zero in every stage
     for (int st = 0; st < S; ++st)
       for (uint32_t o = threadIdx.x * 16u; o < BPS * Cfg::kVBytes; o += blockDim.x * 16u)
         *reinterpret_cast<uint4*>(smem + st * SB + kVOff + o) = make_uint4(0, 0, 0, 0);
-    fence_proxy_async_smem();
   }
+  fence_proxy_async_smem();
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), 512);
     tmem_relinquish();
@@ -510,10 +519,10 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           const int nb = min(BPS, s.nkc - kc);  // a ragged last stage holds fewer chunks
           const uint32_t vfb = smem_u32(&vfull[st]);
           if (FUSED) {
-            mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * kTileBytes);
+            mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * wbox);
             if (tr.is_k) mbar_arrive_expect_tx(vfb, static_cast<uint32_t>(nb) * Cfg::kFBytes);
           } else {
-            mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * (tr.is_k ? kTileBytes + Cfg::kVBytes : kTileBytes));
+            mbar_arrive_expect_tx(fb, static_cast<uint32_t>(nb) * (tr.is_k ? wbox + Cfg::kVBytes : wbox));
           }
 #pragma unroll
           for (int b = 0; b < BPS; ++b) {

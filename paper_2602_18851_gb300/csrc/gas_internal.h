@@ -38,7 +38,10 @@ struct Shape {
   int f16;        // weights (and the MMA operands) are binary16 instead of bf16
   int cols;       // GPT-2 Conv1D layout: element (row r, column c) at w[c * ld + r]
   int f32;        // fp32 weights (CUDA-core back ends only)
-  int tc;         // d_h in {64, 128}: the tensor-core back ends apply
+  int tc;         // d_h in {64, 80, 96, 128}: the tensor-core back ends apply
+  int rows;       // weight rows per head as stored (the model's d_h).  The tensor-core
+                  // kernels get a shape whose dh is the tile head width (64, or 128 for
+                  // d_h 80 / 96 / 128); a head's rows past `rows` read as zero in the tile
 };
 
 // Element offset of row r (head r / d_h, row r % d_h inside it) of a weight matrix.

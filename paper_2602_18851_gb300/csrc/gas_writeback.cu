@@ -106,6 +106,13 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
   // Rows and K ranges of Y that no head uses stay zero for the whole launch.
   for (uint32_t o = threadIdx.x * 16u; o < 2u * YB; o += kWbThreads * 16u)
     *reinterpret_cast<uint4*>(ybuf_s + o) = make_uint4(0, 0, 0, 0);
+  // A d_h 80 / 96 head fills only the top d_h rows (K) of its box; the rest stay zero.
+  const uint32_t wbox = cols ? kBox : static_cast<uint32_t>((128 / DH) * a.s.rows) * 128u;
+  if (wbox < kBox)
+    for (int st = 0; st < S; ++st)
+      for (int b = 0; b < 2; ++b)
+        for (uint32_t o = wbox + threadIdx.x * 16u; o < kBox; o += kWbThreads * 16u)
+          *reinterpret_cast<uint4*>(ring + st * kStage + b * kBox + o) = make_uint4(0, 0, 0, 0);
   fence_proxy_async_smem();
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), Cfg::kTmemCols);
@@ -130,7 +137,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
           if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1u, abort, a.status)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full[st]);
           const uint32_t dst = smem_u32(ring + st * kStage);
-          mbar_arrive_expect_tx(fb, kStage);
+          mbar_arrive_expect_tx(fb, 2u * wbox);
           if (cols) {
             // Conv1D: box b holds rows (K) 64b.. of the tile for the 128 columns (M),
             // K-major, fetched as two 64-column halves of 64-row boxes

@@ -83,6 +83,9 @@ WORKLOADS = {
     "tiny-dh80": Workload("tiny-dh80", 2, 320, 4, 2, 80, 10, "spike4", _BASE_SEED + 18),
     "tiny-dh96": Workload("tiny-dh96", 2, 384, 6, 3, 96, 10, "lognormal", _BASE_SEED + 19),
     "tiny-dh256": Workload("tiny-dh256", 2, 512, 4, 2, 256, 10, "spike1", _BASE_SEED + 20),
+    # A full-size model with d_h 80 (Phi-2-like: 32 layers, d 2560, 32/32 heads), for
+    # timing the tensor-core back ends on a head width that does not fill 128-row tiles.
+    "dh80-mha": Workload("dh80-mha", 32, 2560, 32, 32, 80, 30, "spike4", _BASE_SEED + 22),
 }
 
 # Transient recipe (per step, per weight matrix W of one head or KV group):

@@ -27,7 +27,7 @@ def _inputs(wl):
     return wq, wk, make_start_vectors(wl, device="cuda")
 
 
-@pytest.mark.parametrize("name", ["tiny-gqa128", "tiny-gqa", "ragged128", "gpt2-small", "tiny-g32"])
+@pytest.mark.parametrize("name", ["tiny-gqa128", "tiny-gqa", "ragged128", "gpt2-small", "tiny-g32", "tiny-dh96"])
 @pytest.mark.parametrize("method", ["fused", "gram", "stream"])
 def test_f16_weights_match_oracle(f16_oracle, name, method):
     wl = get_workload(name)

@@ -1,7 +1,9 @@
-"""Head widths outside {64, 128} (80, 96, 256) and fp32 weights: the streaming back end
-and the whole-layer path against the oracle (and, for fp32 values that bf16 cannot
-hold, against the dense-SVD closed form of the finite-k estimate); the tensor-core
-back ends refuse them cleanly."""
+"""Head widths outside {64, 128} (80, 96, 256) and fp32 weights against the oracle (and,
+for fp32 values that bf16 cannot hold, against the dense-SVD closed form of the finite-k
+estimate).  d_h 80 and 96 run on every back end (the tensor-core ones place a head in a
+128-row tile whose remaining rows are zero); d_h 256 and fp32 weights run on the
+streaming back end and the whole-layer path, and the tensor-core back ends refuse them
+cleanly."""
 
 import numpy as np
 import pytest
@@ -17,25 +19,47 @@ from tests.parity_utils import (SIGMA_RTOL, V_ATOL, assert_sigma_close, assert_v
 pytestmark = pytest.mark.gpu
 
 
+@pytest.mark.parametrize("method", ["auto", "fused", "gram", "stream"])
 @pytest.mark.parametrize("name", ["tiny-dh80", "tiny-dh96", "tiny-dh256"])
-def test_other_head_widths_match_oracle(name):
+def test_other_head_widths_match_oracle(name, method):
     wl = get_workload(name)
     wq, wk, v_in, _ = gpu_inputs(wl)
+    tensor_cores = wl.d_h in (80, 96)
     with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
-        sigma, s, v_out = h.refresh(wq, wk, wl.iters, v_in)  # AUTO: the streaming back end
-        torch.cuda.synchronize()
-        assert h.device_status(clear=True) == 0
-        assert h.last_launch_names()[0].startswith("stream")
-        for m in ("fused", "gram"):
-            h.set_method(m)
+        h.set_method(method)
+        if method in ("fused", "gram") and not tensor_cores:
             with pytest.raises(gas.GasError) as e:
                 h.refresh(wq, wk, 2, v_in)
             assert e.value.status == gas.GAS_ERR_UNSUPPORTED
+            return
+        sigma, s, v_out = h.refresh(wq, wk, wl.iters, v_in)
+        torch.cuda.synchronize()
+        assert h.device_status(clear=True) == 0
+        if method == "auto":  # AUTO picks the fused tensor-core back end where it applies
+            assert h.last_launch_names()[0].startswith("gram_fused" if tensor_cores else "stream")
     sig_ref, v_ref = oracle_for(wl, wq, wk, v_in)
     assert_sigma_close(sigma.double().cpu().numpy().ravel(), sig_ref.ravel(), rtol=SIGMA_RTOL)
     assert_v_close(v_out.cpu().numpy().reshape(-1, wl.d), v_ref.reshape(-1, wl.d), atol=V_ATOL)
     np.testing.assert_allclose(s.double().cpu().numpy(), oracle_scales(wl, sig_ref.reshape(wl.layers, wl.n_q)),
                                rtol=1e-3)
+
+
+def test_conv1d_layout_needs_whole_head_tiles():
+    """Conv1D weights are read as 64-row boxes of whole heads: with d_h 80 the tensor-core
+    back ends refuse them, and so does the streaming back end (nn.Linear layout only)."""
+    wl = get_workload("tiny-dh80")
+    rows = wl.n_q * wl.d_h + wl.n_kv * wl.d_h
+    buf = torch.zeros(wl.layers, wl.d, rows, dtype=torch.bfloat16, device="cuda")
+    cq = [buf[l].view(-1) for l in range(wl.layers)]
+    ck = [buf[l].view(-1)[wl.n_q * wl.d_h:] for l in range(wl.layers)]
+    v_in = make_start_vectors(wl, device="cuda")
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        h.set_weight_layout(ld_q=rows, ld_k=rows, layout="cols")
+        for m in ("auto", "fused", "gram", "stream"):
+            h.set_method(m)
+            with pytest.raises(gas.GasError) as e:
+                h.refresh(cq, ck, 2, v_in)
+            assert e.value.status == gas.GAS_ERR_UNSUPPORTED
 
 
 @pytest.mark.parametrize("name", ["tiny-dh96", "tiny-dh256"])

@@ -63,7 +63,7 @@ def _same(a, b):
         assert torch.equal(x, y), (x.flatten()[:4], y.flatten()[:4])
 
 
-@pytest.mark.parametrize("name", ["tiny-gqa128", "ragged128", "tiny-gqa"])
+@pytest.mark.parametrize("name", ["tiny-gqa128", "ragged128", "tiny-gqa", "tiny-dh80"])
 @pytest.mark.parametrize("method", METHODS)
 def test_padded_rows_match_contiguous(name, method):
     wl = get_workload(name)
