@@ -879,13 +879,9 @@ template <int NZ, int DH, bool FUSED, bool GENERIC>
 cudaError_t launch_gram_cfg(const GramArgs& a, int num_sms, cudaStream_t st) {
   using Cfg = GramCfg<NZ, GramBps<NZ, GENERIC>::value, FUSED>;
   auto kern = gram_kernel<NZ, DH, FUSED, GENERIC>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(Cfg::kSmem));
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static unsigned long long configured = 0;  // one bit per device: the attribute is per device
+  cudaError_t e = set_smem_per_device(reinterpret_cast<const void*>(kern), static_cast<int>(Cfg::kSmem), configured);
+  if (e != cudaSuccess) return e;
   const int T = a.s.L * (a.s.tiles_k + a.s.tiles_q);
   const int grid = T < num_sms ? T : num_sms;
   cudaLaunchConfig_t cfg = {};

@@ -172,6 +172,19 @@ struct ScalesArgs {
   float scale_c;
 };
 
+// Raise a kernel's opt-in dynamic shared-memory limit on the current device, once per
+// device (bit `device` of `done`; devices past 63 set it on every call).
+inline cudaError_t set_smem_per_device(const void* kernel, int bytes, unsigned long long& done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = dev < 64 ? 1ull << dev : 0ull;
+  if (bit != 0ull && (done & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done |= bit;
+  return e;
+}
+
 // Launchers (return cudaGetLastError() of the launch).
 cudaError_t launch_stream_pass(const LayerTable& tab, const StreamArgs& a, cudaStream_t st);
 cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st);

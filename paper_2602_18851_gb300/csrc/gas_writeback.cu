@@ -298,13 +298,10 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
 template <int DH, int NZ, bool GENERIC>
 cudaError_t launch_wb_gen(const WbArgs& a, int num_sms, cudaStream_t st) {
   using Cfg = WbCfg<NZ>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(writeback_kernel<DH, NZ, GENERIC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(Cfg::kSmem));
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static unsigned long long configured = 0;  // one bit per device: the attribute is per device
+  cudaError_t e = set_smem_per_device(reinterpret_cast<const void*>(writeback_kernel<DH, NZ, GENERIC>),
+                                      static_cast<int>(Cfg::kSmem), configured);
+  if (e != cudaSuccess) return e;
   const int ncb = (a.s.d + kWbCols - 1) / kWbCols;
   const int T = a.s.L * a.s.tiles_k * ncb;
   const int grid = T < num_sms ? T : num_sms;
