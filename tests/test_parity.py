@@ -11,7 +11,7 @@ import pytest
 import torch
 
 from synth import get_workload, make_start_vectors
-from tests.parity_utils import (assert_sigma_close, assert_v_close, gpu_inputs, oracle_for,
+from tests.parity_utils import (V_ATOL, assert_sigma_close, assert_v_close, gpu_inputs, oracle_for,
                                 oracle_scales, run_library)
 
 pytestmark = pytest.mark.gpu
@@ -217,6 +217,30 @@ def test_start_vector_scale(name, method):
         assert_sigma_close(got["sigma"].ravel(), base["sigma"].ravel(), rtol=1e-4, what="sigma vs unscaled")
         assert_v_close(got["v_out"], base["v_out"].reshape(-1, wl.d), atol=1e-4)
         assert got["status"] == 0
+
+
+# v_out bound of the Gram back ends on the 512-layer case.  They iterate with G = A A^T,
+# whose fp32 rounding is relative to ||A||^2: a finite-k iterate that still lies mostly in
+# small singular directions (start vectors nearly orthogonal to the top singular vector,
+# slow spectra) is perturbed by about eps * kappa^2 instead of the streaming back end's
+# eps * kappa.  sigma, the method's output, stays within 1.5e-4 of the oracle there.
+V_ATOL_GRAM_ILL = 1e-2
+
+
+@pytest.mark.parametrize("method", METHODS)
+def test_maximum_layer_count(method):
+    """512 layers, the most one handle takes (one pointer table per launch): every head
+    against the oracle, on a narrow shape (d 64, one 64-column chunk), at k = 6.  Among
+    the 4096 heads a few converge slowly from start vectors nearly orthogonal to the top
+    singular vector (component ~0.01, sigma_2/sigma_1 ~ 0.9)."""
+    wl = get_workload("tiny-gqa").scaled(layers=512, d=64)
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    got = run_library(wl, wq, wk, v_in, method=method, iters=6)
+    sig, v = oracle_for(wl, wq, wk, v_in, iters=6)
+    assert_sigma_close(got["sigma"].ravel(), sig)
+    assert_v_close(got["v_out"], v, atol=V_ATOL if method == "stream" else V_ATOL_GRAM_ILL)
+    assert_sigma_close(got["s"], oracle_scales(wl, sig.reshape(wl.layers, wl.n_q)), what="scale")
+    assert got["status"] == 0
 
 
 @pytest.mark.parametrize("method", METHODS)
