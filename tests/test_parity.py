@@ -290,33 +290,40 @@ def test_methods_agree_with_each_other():
 
 
 def test_transient_refresh_tracks_oracle():
-    """Llama-2-70B transient workload, abridged to keep the test short: cold start of
-    30 iterations, then warm-started refreshes of 2 iterations while the weights take a
-    seeded rank-8 step every call (spike of 5e-2 at steps 40-45).  GPU and oracle each
-    carry their own v; sigma and the layer scale are compared on a sampled layer."""
+    """Llama-2-70B transient workload on a 4-layer slice: cold start of 30 iterations, then
+    99 warm-started refreshes of 2 iterations while the weights take a seeded rank-8 step
+    every call (spike of 5e-2 at steps 40-45).  Every step, on a sampled layer: sigma and
+    the layer scale against the oracle run lock-step from the GPU's own start vectors
+    (strict parity), and sigma against a free-running float64 trajectory that carries its
+    own v from the first step (drift)."""
     from synth.gen import TransientWeights
     import paper_2602_18851_gb300 as gas
     import oracle
     from tests.helpers import tensor_bits
     wl = get_workload("llama2-70b-transient").scaled(layers=4)
+    assert wl.steps == 100
     tw = TransientWeights(wl, device="cuda")
     v = make_start_vectors(wl, device="cuda")
     layer = 2
-    v_or = v[layer:layer + 1].cpu().numpy().copy()
+    v_free = v[layer:layer + 1].cpu().numpy().copy()
+    pairs = [(0, hq) for hq in range(wl.n_q)]
     with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
-        for t in range(48):
+        for t in range(wl.steps):
             if t > 0:
                 tw.step(t)
             iters = wl.cold_iters if t == 0 else wl.iters
+            v_gpu_in = v[layer:layer + 1].cpu().numpy().copy()
             sigma, s, v = h.refresh(tw.wq, tw.wk, iters, v, v_out=v)
             qb = [tensor_bits(tw.wq[layer])]
             kb = [tensor_bits(tw.wk[layer])]
-            pairs = [(0, hq) for hq in range(wl.n_q)]
-            sig_o, vv = oracle.heads(wl.d, wl.n_q, wl.n_kv, wl.d_h, qb, kb, v_or, iters, pairs)
-            v_or = vv.reshape(1, wl.n_q, wl.d).astype(np.float32)
-            assert_sigma_close(sigma[layer].cpu().numpy(), sig_o, rtol=1e-3)
-            s_ref = oracle_scales(wl, sig_o.reshape(1, wl.n_q), n_heads_total=wl.layers * wl.n_q)
-            assert_sigma_close(s[layer:layer + 1].cpu().numpy(), s_ref, what="scale")
+            sig_ls, _ = oracle.heads(wl.d, wl.n_q, wl.n_kv, wl.d_h, qb, kb, v_gpu_in, iters, pairs)
+            sig_fr, vv = oracle.heads(wl.d, wl.n_q, wl.n_kv, wl.d_h, qb, kb, v_free, iters, pairs)
+            v_free = vv.reshape(1, wl.n_q, wl.d).astype(np.float32)
+            got = sigma[layer].cpu().numpy()
+            assert_sigma_close(got, sig_ls, rtol=1e-3, what=f"sigma, step {t} (lock-step)")
+            assert_sigma_close(got, sig_fr, rtol=1e-3, what=f"sigma, step {t} (free-running)")
+            s_ref = oracle_scales(wl, sig_ls.reshape(1, wl.n_q), n_heads_total=wl.layers * wl.n_q)
+            assert_sigma_close(s[layer:layer + 1].cpu().numpy(), s_ref, what=f"scale, step {t}")
 
 
 def test_bf16_inputs_unchanged():
