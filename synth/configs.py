@@ -86,6 +86,9 @@ WORKLOADS = {
     # A full-size model with d_h 80 (Phi-2-like: 32 layers, d 2560, 32/32 heads), for
     # timing the tensor-core back ends on a head width that does not fill 128-row tiles.
     "dh80-mha": Workload("dh80-mha", 32, 2560, 32, 32, 80, 30, "spike4", _BASE_SEED + 22),
+    # A full-size model with d_h 256 (Gemma-7B-like: 28 layers, d 3072, 16/16 heads), for
+    # timing the streaming back end that such head widths run on.
+    "dh256-mha": Workload("dh256-mha", 28, 3072, 16, 16, 256, 30, "spike4", _BASE_SEED + 23),
 }
 
 # Transient recipe (per step, per weight matrix W of one head or KV group):
