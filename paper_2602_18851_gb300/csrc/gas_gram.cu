@@ -156,7 +156,7 @@ __device__ __forceinline__ TileRef decode_tile(const Shape& s, int D, int t) {
 // Shared scratch of the fused epilogue.  `stage` carries one TMEM lane quarter (32 rows)
 // of a query tile's G_Q at a time from the row-per-thread layout tcgen05.ld produces to
 // the block layout of the iteration; xs / ts hold the current x and t' of each head
-// slot (two heads per tile when d_h = 64); red the per-warp partial dot products.
+// slot (two heads per tile when d_h = 64).
 // Layout of a 4-float chunk q of a 128-float row inside a "plane" array: chunks that the
 // lanes of a half-warp read together (same plane, consecutive q / 2 ... see plane_off)
 // are contiguous, so 128-bit shared loads and stores are free of bank conflicts.
@@ -164,7 +164,6 @@ struct EpiSmem {
   float stage[2][32][68];  // [plane][row][16 chunks x 4 floats + 4 pad]
   float xs[2][2][64];      // [slot][plane][64]: x in the same plane layout
   float ts[2][2][64];
-  float red[2][2][8];      // [slot][which dot][warp of the head group]
   int ok[2];
 };
 
@@ -205,25 +204,11 @@ __device__ __forceinline__ float halfwarp_transpose_reduce8(float (&v)[8], int l
   return v[0];
 }
 
-// Sum of the NW per-warp partials of one head (NW = 4 or 8, 16-byte aligned).
-template <int NW>
-__device__ __forceinline__ float red_sum(const float* r) {
-  const float4 a = *reinterpret_cast<const float4*>(r);
-  float t = (a.x + a.y) + (a.z + a.w);
-  if (NW == 8) {
-    const float4 b = *reinterpret_cast<const float4*>(r + 4);
-    t += (b.x + b.y) + (b.z + b.w);
-  }
-  return t;
-}
-
-// The 8 consecutive entries rb .. rb+7 (rb a multiple of 8) of a vector in the plane layout.
-template <int CPT>
-__device__ __forceinline__ void load_rows8(const float* v, int rb, float (&o)[8]) {
-  const float4 a = *reinterpret_cast<const float4*>(v + vec_off<CPT>(rb));
-  const float4 b = *reinterpret_cast<const float4*>(v + vec_off<CPT>(rb + 4));
-  o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
-  o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
+// Sum over the 16 lanes of a half-warp (all lanes get the total).
+__device__ __forceinline__ float halfwarp_sum(float v) {
+#pragma unroll
+  for (int off = 1; off < 16; off <<= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, off);
+  return v;
 }
 
 // k power iterations for the head(s) of one query tile, in R^{d_h}, run by the 8
@@ -235,9 +220,7 @@ __device__ __forceinline__ void load_rows8(const float* v, int rb, float (&o)[8]
 // With x = c z (c a known scalar, c = 1 for z0) one iteration of Algorithm 2 is
 //   t' = G_Q x,  S1 = x.t' = c^2 sigma^2,  y = t' / sqrt(S1),
 //   w  = G_K y,  S2 = y.w = ||v'||^2,       x <- w,  c <- sqrt(S2),
-// two barriers per iteration.  Each thread's share of a dot product is taken from its
-// 8 row partials before they are reduced (S1 = sum over threads of sum_i x_i part_i),
-// so the dot product's warp sum runs beside the row reduction instead of after it.
+// two barriers per iteration.
 template <int DH>
 __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int idx, uint32_t tacc, int q,
                                               int half, int ew, int lane, EpiSmem* ep, volatile int* abort,
@@ -328,17 +311,32 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
     xs[vec_off<CPT>(th)] = (__ldcg(a.z0 + (hidx * 2) * DH + th) + __ldcg(a.z0 + (hidx * 2 + 1) * DH + th)) * inv;
   }
   named_bar_sync(bar, NTH);
-  const bool writer = (lane & 1) == 0;            // one of the two lanes holding a row total
-  float c = 1.0f, sigma = 0.0f, y = 0.0f, n = 0.0f;
+  const bool writer = (lane & 1) == 0;  // one of the two lanes holding a row total
+  // Each half-warp holds all d_h columns of x (and, after the middle barrier, of t'), so
+  // the dot products S1 = x.t' and S2 = y.w are half-warp sums that overlap the next
+  // matvec.  Inside the loop any normalising factor works as long as S2 and the tracked
+  // scale use the same one: rsqrt(S1) is used, and sigma = sqrt(S1) / sqrt(S2 of the
+  // previous iteration) is formed once, with IEEE operations, after the loop.
+  float c2 = 1.0f, c2_prev = 1.0f, s1_last = 0.0f, inv1 = 0.0f, y = 0.0f;
+  float tv[CPT];
+#pragma unroll
+  for (int k = 0; k < CPT; ++k) tv[k] = 0.0f;
   int ridx = 0;
   for (int it = 0; it < a.iters; ++it) {
-    // t' = G_Q x;  S1 = x . t'
     float xv[CPT];
 #pragma unroll
     for (int k = 0; k < CPT; k += 4) {
       const float4 x4 = *reinterpret_cast<const float4*>(xs + vec_off<CPT>(cb + k));
       xv[k] = x4.x; xv[k + 1] = x4.y; xv[k + 2] = x4.z; xv[k + 3] = x4.w;
     }
+    if (it > 0) {  // S2 of the previous iteration: y.w = inv1 * t'.w, w being this x
+      float q = 0.0f;
+#pragma unroll
+      for (int k = 0; k < CPT; ++k) q = fmaf(tv[k], xv[k], q);
+      const float s2 = halfwarp_sum(q) * inv1;
+      c2 = s2 < 0.0f ? 0.0f : s2;  // rounding can dip below 0; NaN must survive
+    }
+    // t' = G_Q x
     float part[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
@@ -347,52 +345,49 @@ __device__ __forceinline__ void fused_iterate(const GramArgs& a, int layer, int 
       for (int k = 0; k < CPT; ++k) acc0 = fmaf(gq[i][k], xv[k], acc0);
       part[i] = acc0;
     }
-    float rv[8];
-    load_rows8<CPT>(xs, rb, rv);
-    float loc = 0.0f;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) loc = fmaf(rv[i], part[i], loc);
     const float tp = halfwarp_transpose_reduce8(part, lane, ridx);
-    float p = warp_sum(loc);
     const int row = rb + ridx;
     if (writer) ts[vec_off<CPT>(row)] = tp;
-    if (lane == 0) ep->red[hs][0][ewh] = p;
     named_bar_sync(bar, NTH);
-    float s1 = red_sum<NWH>(ep->red[hs][0]);
-    s1 = s1 < 0.0f ? 0.0f : s1;  // rounding can dip below 0; NaN must survive
-    const float rs1 = sqrtf(s1);
-    // zero guards that let a NaN through (x == 0 tests are false for NaN)
-    sigma = c == 0.0f ? 0.0f : rs1 / c;
-    const float inv1 = rs1 == 0.0f ? 0.0f : 1.0f / rs1;
-    // w = G_K y with y = t' / sqrt(S1);  S2 = y . w;  next x = w
+    // S1 = x.t';  w = G_K y with y = t' / sqrt(S1);  next x = w
 #pragma unroll
     for (int k = 0; k < CPT; k += 4) {
       const float4 t4 = *reinterpret_cast<const float4*>(ts + vec_off<CPT>(cb + k));
-      xv[k] = t4.x; xv[k + 1] = t4.y; xv[k + 2] = t4.z; xv[k + 3] = t4.w;
+      tv[k] = t4.x; tv[k + 1] = t4.y; tv[k + 2] = t4.z; tv[k + 3] = t4.w;
     }
+    float q1 = 0.0f;
+#pragma unroll
+    for (int k = 0; k < CPT; ++k) q1 = fmaf(xv[k], tv[k], q1);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       float acc0 = 0.0f;
 #pragma unroll
-      for (int k = 0; k < CPT; ++k) acc0 = fmaf(gk[i][k], xv[k], acc0);
+      for (int k = 0; k < CPT; ++k) acc0 = fmaf(gk[i][k], tv[k], acc0);
       part[i] = acc0;
     }
-    // S2 = y.w = sum_i (t'_i / sqrt(S1)) (G_K t')_i / sqrt(S1)
-    load_rows8<CPT>(ts, rb, rv);
-    loc = 0.0f;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) loc = fmaf(rv[i] * inv1, part[i], loc);
+    float s1 = halfwarp_sum(q1);
+    s1 = s1 < 0.0f ? 0.0f : s1;
+    inv1 = s1 == 0.0f ? 0.0f : rsqrtf(s1);  // zero guard that lets a NaN through
+    s1_last = s1;
+    c2_prev = c2;
     const float wrow = halfwarp_transpose_reduce8(part, lane, ridx) * inv1;
-    p = warp_sum(loc);
     y = tp * inv1;
     if (writer) xs[vec_off<CPT>(row)] = wrow;
-    if (lane == 0) ep->red[hs][1][ewh] = p;
     named_bar_sync(bar, NTH);
-    float s2 = red_sum<NWH>(ep->red[hs][1]) * inv1;
-    s2 = s2 < 0.0f ? 0.0f : s2;
-    n = sqrtf(s2);
-    c = n;
   }
+  // ||v'||^2 of the last iteration (for y / ||v'||), and sigma = ||M v_{k-1}||
+  float n = 0.0f;
+  if (a.iters > 0) {
+    float q = 0.0f;
+#pragma unroll
+    for (int k = 0; k < CPT; k += 4) {
+      const float4 x4 = *reinterpret_cast<const float4*>(xs + vec_off<CPT>(cb + k));
+      q = fmaf(tv[k], x4.x, fmaf(tv[k + 1], x4.y, fmaf(tv[k + 2], x4.z, fmaf(tv[k + 3], x4.w, q))));
+    }
+    const float s2 = halfwarp_sum(q) * inv1;
+    n = sqrtf(s2 < 0.0f ? 0.0f : s2);
+  }
+  const float sigma = c2_prev == 0.0f ? 0.0f : sqrtf(s1_last) / sqrtf(c2_prev);
   if (writer && a.iters > 0) a.ybuf[hidx * DH + rb + ridx] = n == 0.0f ? 0.0f : y / n;
   if (th == 0) {
     a.sigma[hidx] = sigma;
