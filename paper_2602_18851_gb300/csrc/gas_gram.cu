@@ -808,7 +808,11 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
   float z[CPL], y[CPL];
 #pragma unroll
   for (int c = 0; c < CPL; ++c) z[c] = zs[lane * CPL + c];
-  float sigma = 0.0f, inv_n = 0.0f;
+  // The loop normalises with rsqrt: z = c * B v with c = rsqrt(n^2) * sqrt(n^2) of the
+  // previous iteration (1 for z0), so sigma = sqrt(z . t) / c and y / ||v'|| are formed
+  // once, with IEEE operations, after the loop.
+  float inv_n = 1.0f, n2_prev = 1.0f;         // this iteration's c = inv_n * sqrt(n2_prev)
+  float s2_last = 0.0f, in_last = 1.0f, n2_c = 1.0f;
   for (int it = 0; it < a.iters; ++it) {
     // t = G_Q z  (= A u');  sigma^2 = z . t (= ||u'||^2);  y = t / sigma (= A u)
     float part[RPW];
@@ -831,8 +835,10 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
     }
     s2 = warp_sum(s2);
     s2 = s2 < 0.0f ? 0.0f : s2;  // rounding can dip below 0; NaN must survive
-    sigma = sqrtf(s2);
-    const float inv_s = sigma == 0.0f ? 0.0f : 1.0f / sigma;
+    s2_last = s2;
+    in_last = inv_n;
+    n2_c = n2_prev;
+    const float inv_s = s2 == 0.0f ? 0.0f : rsqrtf(s2);  // zero guard that lets a NaN through
 #pragma unroll
     for (int c = 0; c < CPL; ++c) y[c] = t[c] * inv_s;
     // w = G_K y  (= B v');  n^2 = y . w (= ||v'||^2);  z = w / n (= B v)
@@ -854,14 +860,17 @@ __global__ void __launch_bounds__(256) iterate_kernel(const __grid_constant__ It
     }
     n2 = warp_sum(n2);
     n2 = n2 < 0.0f ? 0.0f : n2;
-    const float n = sqrtf(n2);
-    inv_n = n == 0.0f ? 0.0f : 1.0f / n;
+    inv_n = n2 == 0.0f ? 0.0f : rsqrtf(n2);
+    n2_prev = n2;
 #pragma unroll
     for (int c = 0; c < CPL; ++c) z[c] = wv[c] * inv_n;
   }
+  const float cz = in_last * sqrtf(n2_c);
+  const float sigma = cz == 0.0f ? 0.0f : sqrtf(s2_last) / cz;
+  const float ny = sqrtf(n2_prev);
   if (warp == 0) {
 #pragma unroll
-    for (int c = 0; c < CPL; ++c) a.ybuf[hidx * DH + lane * CPL + c] = y[c] * inv_n;
+    for (int c = 0; c < CPL; ++c) a.ybuf[hidx * DH + lane * CPL + c] = ny == 0.0f ? 0.0f : y[c] / ny;
   }
   if (tid == 0) {
     a.sigma[hidx] = sigma;
