@@ -326,6 +326,43 @@ def test_transient_refresh_tracks_oracle():
             assert_sigma_close(s[layer:layer + 1].cpu().numpy(), s_ref, what=f"scale, step {t}")
 
 
+def test_transient_refresh_full_size_sampled_layers():
+    """The same transient workload at its full size, in the launch configuration the
+    benchmark times: all 80 layers of the Llama-2-70B GQA shape, 100 refreshes.  Every
+    step, on layers 0, 39 and 79 (all 64 heads each): sigma and the layer scales against
+    the oracle run lock-step from the GPU's own start vectors.  The per-layer
+    perturbations are seeded by (step, layer), so layers 0-3 also match the 4-layer
+    slice above."""
+    from synth.gen import TransientWeights
+    import paper_2602_18851_gb300 as gas
+    import oracle
+    from tests.helpers import tensor_bits
+    wl = get_workload("llama2-70b-transient")
+    assert wl.layers == 80 and wl.steps == 100
+    tw = TransientWeights(wl, device="cuda")
+    v = make_start_vectors(wl, device="cuda")
+    sample = [0, 39, 79]
+    pairs = [(i, hq) for i in range(len(sample)) for hq in range(wl.n_q)]
+    worst = 0.0
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        for t in range(wl.steps):
+            if t > 0:
+                tw.step(t)
+            iters = wl.cold_iters if t == 0 else wl.iters
+            v_gpu_in = v[sample].cpu().numpy()
+            sigma, s, v = h.refresh(tw.wq, tw.wk, iters, v, v_out=v)
+            qb = [tensor_bits(tw.wq[l]) for l in sample]
+            kb = [tensor_bits(tw.wk[l]) for l in sample]
+            sig, _ = oracle.heads(wl.d, wl.n_q, wl.n_kv, wl.d_h, qb, kb, v_gpu_in, iters, pairs,
+                                  want_v=False)
+            got = sigma[sample].cpu().numpy().ravel()
+            worst = max(worst, assert_sigma_close(got, sig, rtol=1e-3, what=f"sigma, step {t}"))
+            s_ref = oracle_scales(wl, sig.reshape(len(sample), wl.n_q))
+            assert_sigma_close(s[sample].cpu().numpy(), s_ref, what=f"scale, step {t}")
+        assert h.device_status(clear=True) == 0
+    print(f"full-size transient: worst sigma rel err over 100 steps {worst:.2e}")
+
+
 def test_bf16_inputs_unchanged():
     """The library never writes the weights or v_in (when v_out is separate)."""
     import paper_2602_18851_gb300 as gas
