@@ -179,9 +179,10 @@ inline cudaError_t set_smem_per_device(const void* kernel, int bytes, unsigned l
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   const unsigned long long bit = dev < 64 ? 1ull << dev : 0ull;
-  if (bit != 0ull && (done & bit)) return cudaSuccess;
+  // `done` is a per-kernel static shared by every thread of the process: atomic accesses
+  if (bit != 0ull && (__atomic_load_n(&done, __ATOMIC_RELAXED) & bit)) return cudaSuccess;
   e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-  if (e == cudaSuccess) done |= bit;
+  if (e == cudaSuccess) __atomic_fetch_or(&done, bit, __ATOMIC_RELAXED);
   return e;
 }
 
