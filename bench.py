@@ -139,21 +139,28 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
         self.thread.join(timeout=2)
+        return self.summarise(self.lines)
+
+    @staticmethod
+    def summarise(lines):
+        """Median SM clock, maximum clock and power, and the throttle reasons seen active,
+        from `nvidia-smi --query-gpu=<FIELDS> --format=csv,noheader,nounits` lines."""
         sm, smax, power, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        for ln in lines:
             parts = [x.strip() for x in ln.split(",")]
             if len(parts) < 8:
                 continue
-            try:
-                sm.append(float(parts[0]))
-                smax.append(float(parts[1]))
-                power.append(float(parts[2]))
-            except ValueError:
-                continue
-            for n, v in zip(names, parts[4:8]):
+            for n, v in zip(names, parts[4:8]):   # counted even when a clock reads N/A
                 if v.lower().startswith("active"):
                     reasons.add(n)
+            try:
+                vals = [float(x) for x in parts[:3]]
+            except ValueError:
+                continue
+            sm.append(vals[0])
+            smax.append(vals[1])
+            power.append(vals[2])
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
@@ -184,6 +191,11 @@ def profiled_traffic(kernel, units):
     if shas != [m.group(2), m.group(3)]:
         return None
     return int(m.group(1)) * units
+
+
+def needs_l2_flush(input_bytes):
+    """Inputs below twice the L2 size could be re-read from L2 by the next timed step."""
+    return input_bytes < 2 * L2_BYTES
 
 
 def measured_peaks():
@@ -503,7 +515,7 @@ def main():
     # Inputs that fit in L2 (the small GPT-2 shape) would be timed warm: such workloads
     # get an L2 flush (a 512 MB write) before every step, outside that step's events.
     in_bytes = wl.weight_bytes() + v_in.numel() * 4
-    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev) if in_bytes < 2 * L2_BYTES else None
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev) if needs_l2_flush(in_bytes) else None
     step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
