@@ -223,6 +223,18 @@ const char *gas_status_string(gas_status s);
  * word (GAS_DEV_* bits).  Returns GAS_ERR_DEVICE_TIMEOUT when the timeout bit is set. */
 gas_status gas_get_device_status(gas_handle h, int *code, int clear);
 
+/*
+ * Self-test of the device-side failure detection.  Enqueues on `stream` one small
+ * kernel whose bounded wait runs out on purpose, the same wait the Gram and write-back
+ * kernels use: which = 0 waits for an mbarrier phase that nothing completes, which = 1
+ * for a global flag that nothing writes.  After the library's wait limit (2 s) the
+ * kernel sets GAS_DEV_WAIT_TIMEOUT in this handle's device status word and returns;
+ * it holds no tensor memory and leaves no copy in flight, so the context stays usable.
+ * Read the outcome with gas_get_device_status.  Touches no caller buffer.
+ * Errors: GAS_ERR_INVALID_ARG (NULL handle, which not 0 or 1), GAS_ERR_CUDA (launch).
+ */
+gas_status gas_selftest_wait_timeout(gas_handle h, int which, void *stream);
+
 /* Number of kernel launches the last gas_spectral_norms / gas_refresh enqueued. */
 int gas_last_launch_count(gas_handle h);
 

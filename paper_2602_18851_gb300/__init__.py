@@ -98,6 +98,7 @@ def load(path: str = LIB_PATH):
     lib.gas_status_string.argtypes = [c_int]
     lib.gas_status_string.restype = ctypes.c_char_p
     lib.gas_get_device_status.argtypes = [vp, ctypes.POINTER(c_int), c_int]
+    lib.gas_selftest_wait_timeout.argtypes = [vp, c_int, vp]
     lib.gas_last_launch_count.argtypes = [vp]
     lib.gas_set_launch_events.argtypes = [vp, vp, c_int]
     lib.gas_last_launch_name.argtypes = [vp, c_int]
@@ -280,6 +281,11 @@ class Handle:
         if st not in (GAS_OK, GAS_ERR_DEVICE_TIMEOUT):
             _check(st, self._h)
         return code.value
+
+    def selftest_wait_timeout(self, which: int, stream=None) -> None:
+        """Enqueue a kernel whose bounded wait runs out on purpose (0: an mbarrier phase,
+        1: a cross-CTA flag); afterwards device_status() reports GAS_DEV_WAIT_TIMEOUT."""
+        _check(load().gas_selftest_wait_timeout(self._h, int(which), _stream_ptr(stream)), self._h)
 
     # -- compute -------------------------------------------------------------------------
     def _vec_args(self, v_in, v_out, sigma, device):

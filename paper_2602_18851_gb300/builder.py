@@ -16,7 +16,7 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libgas.so")
 
 SOURCES = ["gas_api.cpp", "gas_stream.cu", "gas_gram.cu", "gas_writeback.cu", "gas_static.cu", "gas_layer.cu",
-           "gas_fp8.cu"]
+           "gas_fp8.cu", "gas_selftest.cu"]
 HEADERS = ["gas_device.cuh", "gas_internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]

@@ -848,6 +848,15 @@ gas_status gas_get_device_status(gas_handle h, int* code, int clear) {
   return GAS_OK;
 }
 
+gas_status gas_selftest_wait_timeout(gas_handle h, int which, void* stream) {
+  if (!h) return GAS_ERR_INVALID_ARG;
+  if (which != 0 && which != 1) return fail(h, GAS_ERR_INVALID_ARG, "which must be 0 or 1 (got %d)", which);
+  cudaError_t e = cudaSetDevice(h->device);
+  if (e == cudaSuccess) e = gas::launch_wait_selftest(h->status, which, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "self-test launch");
+  return GAS_OK;
+}
+
 int gas_last_launch_count(gas_handle h) { return h ? h->last_launches : 0; }
 
 gas_status gas_set_launch_events(gas_handle h, void* const* events, int n_events) {

@@ -197,6 +197,7 @@ cudaError_t launch_writeback(const WbArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_layer_rowdot(const LayerTable& tab, const LayerArgs& a, cudaStream_t st);
 cudaError_t launch_layer_coldot(const LayerTable& tab, const LayerArgs& a, cudaStream_t st);
 cudaError_t launch_layer_finalize(const LayerArgs& a, cudaStream_t st);
+cudaError_t launch_wait_selftest(unsigned* status, int which, cudaStream_t st);
 void set_global_error(const char* msg);  // message returned by gas_last_error(NULL)
 size_t gram_smem_bytes(int nz);
 

@@ -289,6 +289,32 @@ def test_methods_agree_with_each_other():
     assert_sigma_close(c["sigma"].ravel(), a["sigma"].ravel(), rtol=1e-5)
 
 
+@pytest.mark.parametrize("which", [0, 1])
+def test_bounded_wait_runs_out_and_context_stays_usable(which):
+    """Failure detection on the device: a wait that nothing completes (an mbarrier phase,
+    or a flag no kernel writes) gives up after the 2 s limit, sets the timeout bit of the
+    status word and returns; the same handle then refreshes correctly."""
+    import time
+    import paper_2602_18851_gb300 as gas
+    wl = get_workload("tiny-gqa128")
+    wq, wk, v_in, _ = gpu_inputs(wl)
+    with gas.Handle(wl.layers, wl.d, wl.n_q, wl.n_kv, wl.d_h) as h:
+        assert h.device_status(clear=True) == 0
+        t0 = time.perf_counter()
+        h.selftest_wait_timeout(which)
+        code = h.device_status(clear=True)      # synchronises: the kernel has returned
+        waited = time.perf_counter() - t0
+        assert code == gas.GAS_DEV_WAIT_TIMEOUT
+        assert 1.5 < waited < 30.0, waited
+        assert h.device_status() == 0           # cleared
+        sigma, s, v_out = h.refresh(wq, wk, wl.iters, v_in)
+        torch.cuda.synchronize()
+        assert h.device_status() == 0
+    sig, v = oracle_for(wl, wq, wk, v_in)
+    assert_sigma_close(sigma.cpu().numpy().ravel(), sig)
+    assert_v_close(v_out.cpu().numpy(), v)
+
+
 def test_transient_refresh_tracks_oracle():
     """Llama-2-70B transient workload on a 4-layer slice: cold start of 30 iterations, then
     99 warm-started refreshes of 2 iterations while the weights take a seeded rank-8 step
