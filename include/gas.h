@@ -224,7 +224,8 @@ const char *gas_status_string(gas_status s);
 gas_status gas_get_device_status(gas_handle h, int *code, int clear);
 
 /*
- * Self-test of the device-side failure detection.  Enqueues on `stream` one small
+ * Self-test of the device-side failure detection (library infrastructure; the paper has
+ * no counterpart).  Enqueues on `stream` one small
  * kernel whose bounded wait runs out on purpose, the same wait the Gram and write-back
  * kernels use: which = 0 waits for an mbarrier phase that nothing completes, which = 1
  * for a global flag that nothing writes.  After the library's wait limit (2 s) the
