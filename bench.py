@@ -42,7 +42,7 @@ L2_BYTES = 129 * 1024 * 1024          # GB300 L2
 L2_FLUSH_BYTES = 512 * 1024 * 1024    # written between timed steps when the inputs fit in L2
 
 METRIC = "full-model sigma+scale refresh ms (Llama-2-70B GQA shape); % of HBM roofline"
-METRIC_LAYER = "whole-layer sigma+scale refresh ms (Algorithms 2-3 as printed); % of HBM roofline of its passes"
+METRIC_LAYER = "whole-layer sigma+scale refresh ms (M = W^Q W^K_exp^T over all heads, Section 4.2); % of HBM roofline of its passes"
 METRIC_E4M3 = "E4M3 cast of one Llama-2-70B layer's attention logits (2x64x1024x1024 bf16) ms; % of HBM roofline"
 
 
@@ -61,7 +61,7 @@ def parse():
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU-baseline sample budget")
     p.add_argument("--path", default="refresh", choices=["refresh", "e4m3", "layer"],
                    help="refresh: per-head sigma + scales (default); layer: whole-layer sigma "
-                        "(Algorithms 2-3 as printed); e4m3: the scales' consumer")
+                        "(M over all heads of a layer, Section 4.2); e4m3: the scales' consumer")
     p.add_argument("--dtype", default="bf16", choices=["bf16", "f16"], help="weight element type")
     p.add_argument("--layout", default="rows", choices=["rows", "padded", "cols"],
                    help="weight storage: nn.Linear rows, rows padded by 64 elements, GPT-2 Conv1D")
@@ -168,29 +168,28 @@ class ClockSampler:
 
 
 def profiled_traffic(kernel, units):
-    """DRAM bytes per launch of `kernel` from the committed ncu summary: the profiled
-    bytes per unit (a layer of the refresh, a whole logits tensor of the E4M3 cast) times
-    `units` (traffic grows in proportion to the layers).  None when the kernel source
-    changed since the counters were taken."""
+    """DRAM bytes per launch of `kernel` from the committed ncu figures in
+    profiles/traffic.json: the profiled bytes per unit (a layer of the refresh, a whole
+    logits tensor of the E4M3 cast) times `units` (traffic grows in proportion to the
+    layers).  None when the kernel has no figure or its source changed since the
+    counters were taken."""
     import hashlib
-    import re
-    files = {"gram_fused": ("launches_llama2-70b-gqa.md", ["gas_gram.cu", "gas_device.cuh"]),
-             "fp8_quantize": ("fp8_quantize_llama2-70b-layer-logits.md", ["gas_fp8.cu", "gas_device.cuh"])}
-    if kernel not in files:
-        return None
-    name, srcs = files[kernel]
     try:
-        text = open(os.path.join(ROOT, "profiles", name)).read()
-    except OSError:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f).get(kernel)
+    except (OSError, ValueError):
         return None
-    m = re.search(r"traffic_bytes_per_(?:layer|launch)=(\d+) source_sha1=(\w+) device_sha1=(\w+)", text)
-    if not m:
+    if not isinstance(rec, dict) or "bytes_per_unit" not in rec:
         return None
     csrc = os.path.join(ROOT, "paper_2602_18851_gb300", "csrc")
-    shas = [hashlib.sha1(open(os.path.join(csrc, f), "rb").read()).hexdigest() for f in srcs]
-    if shas != [m.group(2), m.group(3)]:
-        return None
-    return int(m.group(1)) * units
+    for name, sha in rec.get("sources", {}).items():
+        try:
+            with open(os.path.join(csrc, name), "rb") as f:
+                if hashlib.sha1(f.read()).hexdigest() != sha:
+                    return None
+        except OSError:
+            return None
+    return int(rec["bytes_per_unit"]) * units
 
 
 def needs_l2_flush(input_bytes):
@@ -211,12 +210,27 @@ def measured_peaks():
 # ------------------------------------------------------------------------------------
 # CPU baseline: the float64 oracle on a bounded sample of the same workload
 # ------------------------------------------------------------------------------------
-def oracle_sample_ms(wl, iters, budget_s, wq=None, wk=None, v_in=None):
-    """Time the oracle (factored form, all host cores) on whole layers of the workload
-    until about `budget_s` seconds of CPU work; extrapolate to a full refresh."""
-    import oracle
+def _layer_bits(wl, layer, wq=None, wk=None):
+    """uint16 bit patterns of one layer's weights: the bench's own tensors when given,
+    else the same seeded draw on the host."""
     from synth.gen import _draw_layer
-    threads = oracle.max_threads()
+    if wq is not None:
+        qb = wq[layer].cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+        kb = wk[layer].cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+    else:
+        q, k, _ = _draw_layer(wl, layer, "cpu", wl.seed)
+        qb = q.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+        kb = k.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    return qb, kb
+
+
+def oracle_sample_ms(wl, iters, budget_s, wq=None, wk=None, v_in=None, threads=0, mode="factored",
+                     max_heads=None):
+    """Time the oracle on whole layers of the workload (or on the first `max_heads` heads
+    of layer 0) until about `budget_s` seconds of CPU work; extrapolate to a full refresh.
+    threads = 0 uses every host core (OpenMP over heads); mode "explicit" forms each M_h."""
+    import oracle
+    nthr = oracle.max_threads() if threads <= 0 else threads
     if v_in is None:
         v_np = make_start_vectors(wl, device="cpu").numpy()
     else:
@@ -224,29 +238,46 @@ def oracle_sample_ms(wl, iters, budget_s, wq=None, wk=None, v_in=None):
     spent, heads, layers_done = 0.0, 0, 0
     layer = 0
     while layer < wl.layers and (spent < budget_s or layers_done == 0):
-        if wq is not None:
-            qb = wq[layer].cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
-            kb = wk[layer].cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
-        else:
-            q, k, _ = _draw_layer(wl, layer, "cpu", wl.seed)
-            qb = q.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
-            kb = k.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+        qb, kb = _layer_bits(wl, layer, wq, wk)
         qs = [None] * wl.layers
         ks = [None] * wl.layers
         qs[layer], ks[layer] = qb, kb
-        pairs = [(layer, h) for h in range(wl.n_q)]
+        n = wl.n_q if max_heads is None else min(wl.n_q, max_heads)
+        pairs = [(layer, h) for h in range(n)]
         t0 = time.perf_counter()
-        oracle.heads(wl.d, wl.n_q, wl.n_kv, wl.d_h, qs, ks, v_np, iters, pairs, want_v=True)
+        oracle.heads(wl.d, wl.n_q, wl.n_kv, wl.d_h, qs, ks, v_np, iters, pairs, want_v=True, mode=mode,
+                     threads=nthr)
         spent += time.perf_counter() - t0
         heads += len(pairs)
         layers_done += 1
         layer += 1
+        if max_heads is not None:
+            break
     per_head_s = spent / heads
     full_ms = per_head_s * wl.heads * 1e3
-    return {"value": full_ms, "unit": "ms", "cores": threads, "kind": "oracle",
-            "sample": f"{heads} heads ({layers_done} whole layers) of {wl.name}, {iters} iterations, "
-                      f"float64 factored power iteration incl. v write-back, {spent:.1f} s; "
-                      f"extrapolated linearly to all {wl.heads} heads"}
+    what = f"{layers_done} whole layers" if max_heads is None else f"heads 0-{heads - 1} of layer 0"
+    form = ("float64 factored power iteration incl. v write-back" if mode == "factored" else
+            "float64 power iteration on the explicitly formed d x d M_h incl. forming it")
+    return {"value": full_ms, "unit": "ms", "cores": nthr, "kind": "oracle",
+            "sample": f"{heads} heads ({what}) of {wl.name}, {iters} iterations, {form}, {spent:.1f} s "
+                      f"on {nthr} thread(s); extrapolated linearly to all {wl.heads} heads"}
+
+
+def cpu_baseline(wl, iters, budget_s, wq=None, wk=None, v_in=None):
+    """The oracle as it stands: the factored form on every host core (the reported value),
+    the same form on one core, and the explicit-M form on one head per core."""
+    import oracle
+    out = oracle_sample_ms(wl, iters, budget_s, wq=wq, wk=wk, v_in=v_in)
+    single = oracle_sample_ms(wl, iters, budget_s / 3, wq=wq, wk=wk, v_in=v_in, threads=1)
+    nthr = oracle.max_threads()
+    explicit = oracle_sample_ms(wl, iters, 0.0, wq=wq, wk=wk, v_in=v_in, mode="explicit",
+                                max_heads=min(wl.n_q, nthr))
+    # heads run in parallel, one per thread: the all-heads estimate divides by the threads
+    if min(wl.n_q, nthr) < nthr:
+        explicit["value"] *= min(wl.n_q, nthr) / nthr
+    out["single_thread"] = {"value": single["value"], "cores": 1, "sample": single["sample"]}
+    out["explicit"] = {"value": explicit["value"], "cores": explicit["cores"], "sample": explicit["sample"]}
+    return out
 
 
 def arrange_weights(h, wl, wq, wk, layout):
@@ -559,7 +590,7 @@ def main():
     algo_step = weight_b + 2 * v_b
     method = "fused" if "gram_fused" in names else ("gram" if "gram" in names else "stream")
     if args.path == "layer":
-        # Algorithms 2-3 as printed: four weight passes per iteration (k_rowdot, q_coldot,
+        # whole-layer M (Section 4.2): four weight passes per iteration (k_rowdot, q_coldot,
         # q_rowdot, k_coldot); the least such a k-step run moves is those passes
         method = "layer"
         v_b = 4 * wl.layers * wl.d
@@ -620,7 +651,7 @@ def main():
     cpu = None
     if (rank == 0 and world == 1 and not args.no_cpu_baseline and args.path == "refresh"
             and args.layout == "rows" and args.dtype == "bf16"):
-        cpu = oracle_sample_ms(wl, iters, args.cpu_seconds, wq=wq, wk=wk, v_in=v_in)
+        cpu = cpu_baseline(wl, iters, args.cpu_seconds, wq=wq, wk=wk, v_in=v_in)
 
     if rank == 0:
         out = {

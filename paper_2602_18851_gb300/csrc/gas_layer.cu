@@ -1,10 +1,14 @@
-// Whole-layer spectral norm: Algorithms 2-3 (Appendix E) exactly as printed, with one
-// persistent v per layer and M = W^Q W^K_exp^T summed over all heads (Section 4.2):
+// Whole-layer spectral norm (Section 4.2, Appendix E): sigma_l = ||M||_2 for the layer's
+// full interaction matrix M = W^Q W^K_exp^T, every query head at once, by power iteration
+// on M with one persistent v per layer.  W^K_exp = W^K R^T, where R (n_q d_h x n_kv d_h)
+// repeats each KV group's d_h coordinates for its G query heads, so W^K is never expanded:
 //
-//   z_kv = W^K^T v           rowdot over Wk          (n_kv*d_h values)
-//   u'   = W^Q RepeatBlocks(z_kv)   coldot over Wq    (d values)
-//   y    = W^Q^T (u'/||u'||)  rowdot over Wq          (n_q*d_h values)
-//   v'   = W^K SumGroups(y)   coldot over Wk          (d values)
+//   M v   = W^Q (R (W^K^T v)):   a row-dot pass over Wk (n_kv*d_h values), the G-fold
+//                                repeat, then a column-sum pass over Wq (d values)
+//   M^T u = W^K (R^T (W^Q^T u)): a row-dot pass over Wq (n_q*d_h values), R^T sums the G
+//                                query blocks of each group, then a column-sum pass over Wk
+//
+// with sigma = ||M v|| and v <- M^T u / ||M^T u|| for u = M v / ||M v||.
 //
 // In the nn.Linear layout Wq[r][c] (r < n_q*d_h, c < d) is W^Q[c][r], so W^Q^T x is a row
 // dot product and W^Q z a column sum.  The z-space has n_q*d_h dimensions, too many for

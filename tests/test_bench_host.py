@@ -71,3 +71,12 @@ def test_cpu_baseline_sample_is_bounded_and_labelled():
     c = bench.oracle_sample_ms(wl, wl.iters, budget_s=0.0)
     assert c["kind"] == "oracle" and c["unit"] == "ms" and c["cores"] >= 1 and c["value"] > 0
     assert "1 whole layers" in c["sample"] and wl.name in c["sample"]
+
+
+def test_cpu_baseline_reports_all_cores_one_core_and_explicit():
+    wl = get_workload("tiny-gqa128")
+    c = bench.cpu_baseline(wl, wl.iters, budget_s=0.0)
+    assert c["kind"] == "oracle" and c["value"] > 0 and c["cores"] >= 1
+    assert c["single_thread"]["cores"] == 1 and c["single_thread"]["value"] > 0
+    assert "1 thread" in c["single_thread"]["sample"]
+    assert c["explicit"]["value"] > 0 and "explicitly formed" in c["explicit"]["sample"]

@@ -1,5 +1,5 @@
-"""GPU parity of the whole-layer sigma (Algorithms 2-3 as printed: one v per layer,
-M = W^Q W^K_exp^T over all heads) against the float64 oracle's Algorithm 3."""
+"""GPU parity of the whole-layer sigma (Section 4.2: one v per layer, M = W^Q W^K_exp^T
+over all heads) against the float64 oracle's Algorithm 3."""
 
 import numpy as np
 import pytest
