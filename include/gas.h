@@ -143,10 +143,11 @@ gas_status gas_refresh(gas_handle h, const void *const *wq, const void *const *w
                        double delta_star, double r_max, float *s, void *stream);
 
 /*
- * Whole-layer spectral norm, Algorithms 2-3 (Appendix E) as printed: one persistent v
- * per layer and M = W^Q W^K_exp^T with W^Q = all n_q heads ([d x n_q*d_h]) and W^K_exp
- * the RepeatBlocks expansion of W^K (Section 4.2, never formed: RepeatBlocks / SumGroups
- * act on the n_kv*d_h-vectors).  sigma_l = ||u'|| of the last iteration.
+ * Whole-layer spectral norm (Section 4.2, Appendix E): sigma_l = ||M||_2 for
+ * M = W^Q W^K_exp^T with W^Q = all n_q heads ([d x n_q*d_h]) and W^K_exp = W^K with each
+ * KV group repeated for its query heads (never formed: the repeat and its transpose, a
+ * sum over each group's query blocks, act on the n_kv*d_h-vectors).  Power iteration
+ * with one persistent v per layer; sigma_l = ||M v|| of the last iteration.
  *   v_in, v_out : device fp32 [layers][d] (v_out may alias v_in or be NULL).
  *   sigma       : device fp32 [layers].
  *   s           : device fp32 [layers] or NULL; if given, the layer scale of Eq. 15 with
@@ -266,21 +267,36 @@ const char *gas_last_launch_name(gas_handle h, int i);
  * library routine: its scratch is a file-scope device array of
  * GAS_STATIC_SCRATCH_BYTES that every GPU loading the library holds until the
  * process exits.
- *   Arguments: as gas_create's shape plus gas_spectral_norms' buffers (wq, wk host
- *   arrays of device pointers; v_in, v_out, sigma device fp32; v_out may be NULL or
- *   alias v_in).  Scratch needed: 2*align256(layers*n_q*ceil(d/256)*d_h*4) +
- *   2*align256(layers*n_q*ceil(d/256)*4) bytes (e.g. 16.8 MB for 32 layers, d 4096,
- *   32 heads, d_h 128); larger shapes are rejected with GAS_ERR_UNSUPPORTED.
+ *   Arguments: layers, d, n_q, n_kv, d_h as for gas_create, with narrower limits:
+ *   d_h 64 or 128, d % 8 == 0, layers <= 512.  Weights are bf16 in the default
+ *   contiguous nn.Linear layout ([n_q*d_h, d] and [n_kv*d_h, d] row-major; no row or
+ *   head stride, no Conv1D layout, no fp16 / fp32).  wq, wk: host arrays of device
+ *   pointers (16-byte aligned); v_in, v_out, sigma: device fp32 as for
+ *   gas_spectral_norms (v_out may be NULL or alias v_in).
+ *   Scratch needed: gas_static_scratch_bytes(layers, d, n_q, d_h), that is, with
+ *   nch = ceil(d / 256) and a(x) = x rounded up to a multiple of 256:
+ *     2*a(layers*n_q*nch*d_h*4) + 2*a(layers*n_q*nch*4) + 2*a(layers*n_q*d_h*4)
+ *     + 3*a(layers*n_q*4) bytes
+ *   (17,969,152 bytes for 32 layers, d 4096, 32 heads, d_h 128).  Shapes that need
+ *   more than GAS_STATIC_SCRATCH_BYTES are rejected with GAS_ERR_UNSUPPORTED before
+ *   any device work.
  *   Errors: as gas_spectral_norms; gas_last_error(NULL) holds the message.
- * The first call on each device looks up the array's device address
- * (cudaGetSymbolAddress) and caches it; make that first call before any stream
- * capture.  All calls share the array and it keeps the last call's contents: calls
- * whose kernels overlap on the GPU (other streams, other threads) race on it.
+ * Every call looks up the array's device address in the current context
+ * (cudaGetSymbolAddress), so the address stays right after cudaDeviceReset or under
+ * another context.  The first call on a device also loads the library's device code:
+ * make that first call before any stream capture.  All calls share the array and it
+ * keeps the last call's contents; each call clears the part that must start at zero
+ * (the reduction counters) on its stream.  Calls whose kernels overlap on the GPU
+ * (other streams, other threads) race on the array.
  */
 #define GAS_STATIC_SCRATCH_BYTES (32u * 1024u * 1024u)
 gas_status gas_spectral_norms_static(int layers, int d, int n_q, int n_kv, int d_h,
                                      const void *const *wq, const void *const *wk, int iters,
                                      const float *v_in, float *v_out, float *sigma, void *stream);
+
+/* Scratch bytes gas_spectral_norms_static needs for a shape (the expression above; 0
+ * when a size is not positive).  Host only; no device work. */
+size_t gas_static_scratch_bytes(int layers, int d, int n_q, int d_h);
 
 #ifdef __cplusplus
 }

@@ -104,6 +104,8 @@ def load(path: str = LIB_PATH):
     lib.gas_last_launch_name.argtypes = [vp, c_int]
     lib.gas_last_launch_name.restype = ctypes.c_char_p
     lib.gas_spectral_norms_static.argtypes = [c_int] * 5 + [vp, vp, c_int, vp, vp, vp, vp]
+    lib.gas_static_scratch_bytes.argtypes = [c_int] * 4
+    lib.gas_static_scratch_bytes.restype = ctypes.c_size_t
     lib.gas_layer_refresh.argtypes = [vp, vp, vp, c_int, vp, vp, vp, c_double, c_double, c_double, vp, vp]
     lib.gas_set_weight_layout.argtypes = [vp, c_int, c_ll, c_ll, c_ll, c_ll]
     lib.gas_set_weight_dtype.argtypes = [vp, c_int]

@@ -13,7 +13,6 @@
 // holds kStaticScratchBytes for it until the process exits.  All calls share it, so
 // calls whose kernels overlap on the GPU (two streams, two host threads) race on it.
 
-#include <atomic>
 #include <cstdio>
 #include <cstring>
 
@@ -24,26 +23,35 @@ namespace gas {
 namespace {
 
 constexpr size_t kStaticScratchBytes = GAS_STATIC_SCRATCH_BYTES;
-constexpr int kMaxDevices = 64;
 
 // Host code must not use this name as a device address (see static_scratch_ptr).
 __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-std::atomic<void*> g_scratch_ptr[kMaxDevices];
-
 size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
-// Device address of the scratch array on the current device, looked up once per device
-// (the first call on a device does this; it should come before any stream capture).
-cudaError_t static_scratch_ptr(int dev, void** out) {
-  void* p = g_scratch_ptr[dev].load(std::memory_order_acquire);
-  if (p == nullptr) {
-    cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_ptr[dev].store(p, std::memory_order_release);
-  }
-  *out = p;
-  return cudaSuccess;
+// Device address of the scratch array in the current context.  It is looked up on every
+// call: the address belongs to the context that loaded the library's device code, so a
+// cached value would go stale after cudaDeviceReset or under another context.  After the
+// first call on a device (which also loads the device code) the lookup is a table search.
+cudaError_t static_scratch_ptr(void** out) { return cudaGetSymbolAddress(out, g_static_scratch); }
+
+// Bytes of scratch one call needs (0 for sizes that are not positive).
+// Layout: z and t partials [L][n_q][nch][d_h], their squared-norm partials [L][n_q][nch],
+// the chunk sums of both ([L][n_q][d_h] and [L][n_q]) and the passes' ticket counters
+// [L][n_q], each region 256-byte aligned.
+struct StaticLayout {
+  size_t vec, nrm, rvec, rnrm, total;
+};
+StaticLayout static_layout(int layers, int d, int n_q, int d_h) {
+  StaticLayout o{};
+  if (layers < 1 || d < 1 || n_q < 1 || d_h < 1) return o;
+  const size_t nch = (static_cast<size_t>(d) + kStreamChunk - 1) / kStreamChunk;
+  o.vec = static_cast<size_t>(layers) * n_q * nch * d_h * sizeof(float);
+  o.nrm = static_cast<size_t>(layers) * n_q * nch * sizeof(float);
+  o.rvec = static_cast<size_t>(layers) * n_q * d_h * sizeof(float);
+  o.rnrm = static_cast<size_t>(layers) * n_q * sizeof(float);
+  o.total = 2 * align256(o.vec) + 2 * align256(o.nrm) + 2 * align256(o.rvec) + 3 * align256(o.rnrm);
+  return o;
 }
 
 }  // namespace
@@ -84,26 +92,16 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
   s.f16 = 0;
   s.f32 = 0;
   s.tc = 1;
-  // Scratch: z and t partials [L][n_q][nch][d_h], their squared-norm partials [L][n_q][nch],
-  // the chunk sums of both ([L][n_q][d_h] and [L][n_q]) and the passes' ticket counters.
-  const size_t vec = static_cast<size_t>(layers) * n_q * s.nch * d_h * sizeof(float);
-  const size_t nrm = static_cast<size_t>(layers) * n_q * s.nch * sizeof(float);
-  const size_t rvec = static_cast<size_t>(layers) * n_q * d_h * sizeof(float);
-  const size_t rnrm = static_cast<size_t>(layers) * n_q * sizeof(float);
-  const size_t need = 2 * gas::align256(vec) + 2 * gas::align256(nrm) + 2 * gas::align256(rvec) +
-                      3 * gas::align256(rnrm);
+  const gas::StaticLayout lay = gas::static_layout(layers, d, n_q, d_h);
+  const size_t vec = lay.vec, nrm = lay.nrm, rvec = lay.rvec, rnrm = lay.rnrm, need = lay.total;
   if (need > gas::kStaticScratchBytes) {
     snprintf(buf, sizeof(buf),
              "gas_spectral_norms_static: this shape needs %zu bytes of scratch, the static array holds %zu",
              need, gas::kStaticScratchBytes);
     return static_fail(GAS_ERR_UNSUPPORTED, buf);
   }
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess || dev < 0 || dev >= gas::kMaxDevices)
-    return static_fail(GAS_ERR_CUDA, "gas_spectral_norms_static: no usable current device");
   void* base = nullptr;
-  e = gas::static_scratch_ptr(dev, &base);
+  cudaError_t e = gas::static_scratch_ptr(&base);
   if (e != cudaSuccess) {
     snprintf(buf, sizeof(buf), "gas_spectral_norms_static: cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
     return static_fail(GAS_ERR_CUDA, buf);
@@ -120,9 +118,17 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
   float* s2r = reinterpret_cast<float*>(r + 2 * gas::align256(rvec) + gas::align256(rnrm));
   unsigned* tickets = reinterpret_cast<unsigned*>(r + 2 * gas::align256(rvec) + 2 * gas::align256(rnrm));
   // Every scratch element a pass reads was written earlier in the same call (each pass
-  // covers all heads, chunks and rows), so nothing has to be cleared between calls.  The
-  // ticket counters start at zero (a device array is zero-initialised when the module
-  // loads) and every pass leaves them at zero again.
+  // covers all heads, chunks and rows), except the ticket counters of the last-CTA
+  // reductions: those must start at zero.  Where they sit depends on the shape, so an
+  // earlier call with another shape may have left partial sums there; they are cleared
+  // on the stream at the start of every call (every pass leaves them at zero again).
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  e = cudaMemsetAsync(tickets, 0, gas::align256(rnrm), st);
+  if (e != cudaSuccess) {
+    snprintf(buf, sizeof(buf), "gas_spectral_norms_static: clearing the ticket counters failed: %s",
+             cudaGetErrorString(e));
+    return static_fail(GAS_ERR_CUDA, buf);
+  }
 
   gas::LayerTable tab;
   std::memset(&tab, 0, sizeof(tab));
@@ -130,7 +136,6 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
     tab.q[l] = static_cast<const uint16_t*>(wq[l]);
     tab.k[l] = static_cast<const uint16_t*>(wk[l]);
   }
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
   gas::StreamArgs a{};
   a.s = s;
   a.mode = gas::kPassK0;
@@ -184,4 +189,8 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
     return static_fail(GAS_ERR_CUDA, buf);
   }
   return GAS_OK;
+}
+
+extern "C" size_t gas_static_scratch_bytes(int layers, int d, int n_q, int d_h) {
+  return gas::static_layout(layers, d, n_q, d_h).total;
 }
