@@ -41,21 +41,31 @@ def test_l2_flush_rule():
 
 
 def test_profiled_traffic_follows_the_kernel_source(tmp_path, monkeypatch):
-    per80 = bench.profiled_traffic("gram_fused", 80)
-    assert per80 is not None and bench.profiled_traffic("gram_fused", 4) * 20 == per80
-    assert bench.profiled_traffic("writeback", 80) is None        # no one-pass figure kept
-    # a copy of the tree whose Gram kernel source differs: the stored counters no longer apply
-    shutil.copytree(os.path.join(ROOT, "profiles"), tmp_path / "profiles")
+    """bench.py reports the stored ncu traffic only while every listed source still has the
+    hash the counters were taken on (checked on a copy of the tree)."""
+    import hashlib
+    import json
     csrc = tmp_path / "paper_2602_18851_gb300" / "csrc"
     csrc.mkdir(parents=True)
-    for f in ("gas_gram.cu", "gas_device.cuh", "gas_fp8.cu"):
+    for f in ("gas_gram.cu", "gas_device.cuh"):
         shutil.copy(os.path.join(ROOT, "paper_2602_18851_gb300", "csrc", f), csrc / f)
+    sha = {f: hashlib.sha1((csrc / f).read_bytes()).hexdigest() for f in ("gas_gram.cu", "gas_device.cuh")}
+    (tmp_path / "profiles").mkdir()
+    (tmp_path / "profiles" / "traffic.json").write_text(json.dumps(
+        {"gram_fused": {"unit": "layer", "bytes_per_unit": 1000, "sources": sha}}))
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.profiled_traffic("gram_fused", 80) == per80
+    assert bench.profiled_traffic("gram_fused", 80) == 80000
+    assert bench.profiled_traffic("gram_fused", 4) == 4000
+    assert bench.profiled_traffic("writeback", 80) is None        # no figure kept
     with open(csrc / "gas_gram.cu", "a") as f:
         f.write("\n// edited\n")
     assert bench.profiled_traffic("gram_fused", 80) is None
-    assert bench.profiled_traffic("fp8_quantize", 1) is not None
+    # the committed file parses, and every entry names its sources
+    with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+        committed = json.load(f)
+    for name, rec in committed.items():
+        if not name.startswith("_"):
+            assert rec["bytes_per_unit"] > 0 and rec["sources"], name
 
 
 def test_measured_peak_is_read_from_the_driver_file():
