@@ -56,6 +56,7 @@ struct gas_ctx {
   float* vn2 = nullptr;          // [L][nq] ||v||^2 of the start vectors (fused kernel)
   unsigned* layer_cnt = nullptr;  // [L] finished heads per layer of the fused kernel
   unsigned* done_cnt = nullptr;   // finished CTAs of the fused kernel
+  unsigned* tile_ctr = nullptr;   // dynamic tile counter of the fused kernel
   unsigned long long* layer_max = nullptr;  // [L] epoch-tagged sigma maxima of the fused kernel
   float* lz = nullptr;           // whole-layer path: z_kv [L][n_kv*d_h]
   float* lu = nullptr;           //                   u'   [L][d]
@@ -253,6 +254,7 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
   a.outr = h->zr;
   a.outr2 = h->n2r;
   a.tickets = h->tickets;
+  a.status = h->status;
   a.v_in = v_in;
   a.s_zero = s_out;
   cudaError_t e = launch(h, "stream_pass_k0", st, [&] { return gas::launch_stream_pass(tab, a, st); });
@@ -269,6 +271,7 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
     q.outr = h->tr;
     q.outr2 = h->s2r;
     q.tickets = h->tickets;
+    q.status = h->status;
     e = launch(h, "stream_pass_q", st, [&] { return gas::launch_stream_pass(tab, q, st); });
     ++launches;
     if (e != cudaSuccess) break;
@@ -285,6 +288,7 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
     k.outr = h->zr;
     k.outr2 = h->n2r;
     k.tickets = h->tickets;
+    k.status = h->status;
     k.v_out = v_out;
     e = launch(h, last ? "stream_pass_kout" : "stream_pass_k", st,
                [&] { return gas::launch_stream_pass(tab, k, st); });
@@ -353,6 +357,7 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
       g.layer_cnt = h->layer_cnt;
       g.layer_max = h->layer_max;
       g.done_cnt = h->done_cnt;
+      g.tile_ctr = h->tile_ctr;
       g.iters = iters;
       g.ybuf = h->ybuf;
       g.sigma = sigma;
@@ -584,7 +589,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_flags = take(L * s.tiles_k * sizeof(unsigned));
   const size_t o_vflags = take(L * s.tiles_k * sizeof(unsigned));
   const size_t o_vn2 = take(L * NQ * 4);
-  const size_t o_lcnt = take((L + 1) * sizeof(unsigned));
+  const size_t o_lcnt = take((L + 2) * sizeof(unsigned));  // head counts, done CTAs, tile counter
   const size_t o_lmax = take(L * sizeof(unsigned long long));
   const size_t o_lz = take(L * static_cast<size_t>(n_kv) * d_h * 4);
   const size_t o_lu = take(L * static_cast<size_t>(d) * 4);
@@ -624,6 +629,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   h->vn2 = reinterpret_cast<float*>(b + o_vn2);
   h->layer_cnt = reinterpret_cast<unsigned*>(b + o_lcnt);
   h->done_cnt = h->layer_cnt + L;
+  h->tile_ctr = h->layer_cnt + L + 1;
   h->layer_max = reinterpret_cast<unsigned long long*>(b + o_lmax);
   h->lz = reinterpret_cast<float*>(b + o_lz);
   h->lu = reinterpret_cast<float*>(b + o_lu);

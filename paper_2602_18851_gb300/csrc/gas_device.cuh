@@ -382,6 +382,16 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32_bmn(int M, int N) {
   return idesc_bf16_f32(M, N) | (1u << 16);
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may start once every CTA of the kernel before it has called
+// griddep_launch_dependents (or exited); griddep_wait then blocks until that kernel has
+// completed and its memory operations are visible.  Without the launch attribute the
+// wait returns at once.
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---------------------------------------------------------------------------------
 // Named barriers, flags, wide tensor-memory loads
 // ---------------------------------------------------------------------------------

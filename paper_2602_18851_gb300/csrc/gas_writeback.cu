@@ -134,6 +134,9 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
         const WbItem w = decode_item(s, t);
         for (int j = 0; j < w.nchunks; ++j) {
           const uint32_t st = issued % S, ph = (issued / S) & 1u;
+          // The first S stages go out at once (W^K does not depend on the previous kernel);
+          // the bounded waits for stages to drain start after that kernel has completed.
+          if (issued == static_cast<uint32_t>(S)) griddep_wait();
           if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1u, abort, a.status)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full[st]);
           const uint32_t dst = smem_u32(ring + st * kStage);
@@ -164,6 +167,7 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
       const uint32_t idesc = idesc_f32acc(128, NZ, f16) | (cols ? 0u : (1u << 15));
       uint32_t consumed = 0, cc = 0, it = 0;
       bool ok = true;
+      griddep_wait();  // its bounded waits start once the previous kernel has completed
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x, ++it) {
         const WbItem w = decode_item(s, t);
         const uint32_t yb = it & 1u;
@@ -246,6 +250,10 @@ __global__ void __launch_bounds__(kWbThreads, 1) writeback_kernel(const __grid_c
     };
     uint32_t cc = 0;
     bool ok = true;
+    // y (and the caller's v_in, which v_out may alias) belong to the kernel launched
+    // before this one: wait until it has completed.  The producer's W^K copies and the
+    // prologue do not depend on it and may already run.
+    griddep_wait();
     // Every stage() is followed by a vote so that all four warps leave together.
     if (blockIdx.x < T) ok = named_bar_and(5, 128, stage(blockIdx.x));
     for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
@@ -305,7 +313,23 @@ cudaError_t launch_wb_gen(const WbArgs& a, int num_sms, cudaStream_t st) {
   const int ncb = (a.s.d + kWbCols - 1) / kWbCols;
   const int T = a.s.L * a.s.tiles_k * ncb;
   const int grid = T < num_sms ? T : num_sms;
-  writeback_kernel<DH, NZ, GENERIC><<<grid, kWbThreads, Cfg::kSmem, st>>>(a);
+  // Programmatic dependent launch: the CTAs may start as the previous kernel's CTAs exit
+  // (only the reads of y wait for that kernel, see griddep_wait).
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kWbThreads);
+  cfg.dynamicSmemBytes = Cfg::kSmem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, writeback_kernel<DH, NZ, GENERIC>, a);
+  if (e == cudaErrorNotSupported || e == cudaErrorInvalidValue) {
+    (void)cudaGetLastError();  // the attribute is refused here: an ordinary stream-ordered launch
+    writeback_kernel<DH, NZ, GENERIC><<<grid, kWbThreads, Cfg::kSmem, st>>>(a);
+  }
   return cudaGetLastError();
 }
 
