@@ -56,7 +56,6 @@ struct gas_ctx {
   float* vn2 = nullptr;          // [L][nq] ||v||^2 of the start vectors (fused kernel)
   unsigned* layer_cnt = nullptr;  // [L] finished heads per layer of the fused kernel
   unsigned* done_cnt = nullptr;   // finished CTAs of the fused kernel
-  unsigned* tile_ctr = nullptr;   // dynamic tile counter of the fused kernel
   unsigned long long* layer_max = nullptr;  // [L] epoch-tagged sigma maxima of the fused kernel
   float* lz = nullptr;           // whole-layer path: z_kv [L][n_kv*d_h]
   float* lu = nullptr;           //                   u'   [L][d]
@@ -357,7 +356,6 @@ gas_status run_gram(gas_ctx* h, const void* const* wq, const void* const* wk, co
       g.layer_cnt = h->layer_cnt;
       g.layer_max = h->layer_max;
       g.done_cnt = h->done_cnt;
-      g.tile_ctr = h->tile_ctr;
       g.iters = iters;
       g.ybuf = h->ybuf;
       g.sigma = sigma;
@@ -589,7 +587,7 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_flags = take(L * s.tiles_k * sizeof(unsigned));
   const size_t o_vflags = take(L * s.tiles_k * sizeof(unsigned));
   const size_t o_vn2 = take(L * NQ * 4);
-  const size_t o_lcnt = take((L + 2) * sizeof(unsigned));  // head counts, done CTAs, tile counter
+  const size_t o_lcnt = take((L + 1) * sizeof(unsigned));
   const size_t o_lmax = take(L * sizeof(unsigned long long));
   const size_t o_lz = take(L * static_cast<size_t>(n_kv) * d_h * 4);
   const size_t o_lu = take(L * static_cast<size_t>(d) * 4);
@@ -629,7 +627,6 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   h->vn2 = reinterpret_cast<float*>(b + o_vn2);
   h->layer_cnt = reinterpret_cast<unsigned*>(b + o_lcnt);
   h->done_cnt = h->layer_cnt + L;
-  h->tile_ctr = h->layer_cnt + L + 1;
   h->layer_max = reinterpret_cast<unsigned long long*>(b + o_lmax);
   h->lz = reinterpret_cast<float*>(b + o_lz);
   h->lu = reinterpret_cast<float*>(b + o_lu);

@@ -40,7 +40,6 @@ struct GramWarps {
 constexpr uint32_t kTileBytes = 128u * 64u * 2u;  // one 128-row x 64-column bf16 box
 constexpr int kSmemBudget = 232448;               // 227 KB opt-in dynamic shared memory
 constexpr int kSmemReserve = 22528;               // alignment slack, barriers, epilogue scratch
-constexpr int kTileQ = 8;                         // slots of the CTA's tile queue
 
 // A ring stage holds BPS consecutive 64-column chunks of a tile: BPS weight boxes, the
 // BPS matching v operand boxes (NZ rows of bf16 hi / lo, key tiles only) and, in the
@@ -427,9 +426,8 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   constexpr uint32_t kFOff = BPS * (kTileBytes + Cfg::kVBytes);  // ... of the fp32 v boxes (fused)
   constexpr int S = Cfg::kStages;
   constexpr uint32_t SB = Cfg::kStageBytes;
-  static_assert(1023 + (4 * S + 2 * Cfg::kAcc + 1 + 2 * kTileQ) * 8 + 8 + 4 * kTileQ + 127 + sizeof(EpiSmem) <=
-                    kSmemReserve,
-                "alignment slack, barriers, tile queue and epilogue scratch must fit in the reserve");
+  static_assert(1023 + (4 * S + 2 * Cfg::kAcc + 1) * 8 + 64 + 127 + sizeof(EpiSmem) <= kSmemReserve,
+                "alignment slack, barriers and epilogue scratch must fit in the reserve");
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment by pointer arithmetic on the shared array itself, so that the
   // compiler keeps every derived pointer in the shared address space.
@@ -443,14 +441,9 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   uint64_t* accf = bars + 4 * S;
   uint64_t* acce = accf + NA;
   uint64_t* done = acce + NA;
-  // Tile queue: the producer claims the tiles and publishes each one (or T, the end) in
-  // slot n % kTileQ; every other role reads the slots in order.
-  uint64_t* tqf = done + 1;        // slot written (producer arrives)
-  uint64_t* tqe = tqf + kTileQ;    // slot read by every consumer thread
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tqe + kTileQ);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  int* tq = reinterpret_cast<int*>(tmem_slot + 2);
-  const uint32_t ep_off = ((smem_u32(tq + kTileQ) + 127u) & ~127u) - smem_u32(smem);
+  const uint32_t ep_off = ((smem_u32(done) + 64u + 127u) & ~127u) - smem_u32(smem);
   EpiSmem* ep = reinterpret_cast<EpiSmem*>(smem + ep_off);
   volatile int no_abort_flag = 0;
 
@@ -470,10 +463,6 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       mbar_init(smem_u32(&acce[i]), NE);
     }
     mbar_init(smem_u32(done), 1);
-    for (int i = 0; i < kTileQ; ++i) {
-      mbar_init(smem_u32(&tqf[i]), 1);
-      mbar_init(smem_u32(&tqe[i]), 1 + NE + 32 * GramWarps<FUSED>::kConvWarps);
-    }
     *abort = 0;
     fence_mbar_init();
   }
@@ -508,15 +497,6 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   const int D = lead_layers(s, gridDim.x);
   // Fused key stages: the conv[] and vfull[] barriers of stage st complete one phase per
   // key-tile use of st; bit st of a role's kpar holds the parity of its next such phase.
-  // Schedule: CTA b takes tiles b, b + gridDim.x, ... below tail0, which keeps every
-  // CTA's mix of key and query tiles (and with it its epilogue load) even.  The fused
-  // kernel hands out the last two waves, tail0 .. T-1, from a global counter (tile
-  // tail0 + n for the n-th claim over all CTAs), so CTAs that are ahead take more of
-  // them and the launch ends together.  Every CTA's tiles increase, so every flag wait
-  // still targets an earlier tile.  The Gram-only kernel strides statically throughout.
-  const int tail0 = T - 2 * static_cast<int>(gridDim.x) > static_cast<int>(gridDim.x)
-                        ? T - 2 * static_cast<int>(gridDim.x)
-                        : static_cast<int>(gridDim.x);
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -524,17 +504,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       const uint64_t pol = l2_policy_evict_first();
       uint32_t issued = 0, kpar = 0u, kmask = 0u;  // kmask bit st: the latest use of st was a key stage
       bool ok = true;
-      int t = static_cast<int>(blockIdx.x);
-      for (uint32_t nt = 0; ok; ++nt) {
-        const uint32_t qs = nt % kTileQ;
-        if (!mbar_wait(smem_u32(&tqe[qs]), ((nt / kTileQ) & 1u) ^ 1u, abort, a.status)) break;
-        tq[qs] = t < T ? t : T;
-        mbar_arrive(smem_u32(&tqf[qs]));
-        if (t >= T) break;
-        // the next tile: static stride, then claimed from the counter in the last waves
-        // (claimed now: its index is first needed after this tile's copies)
-        int next = t + static_cast<int>(gridDim.x);
-        if (FUSED && next >= tail0) next = tail0 + static_cast<int>(atomicAdd(a.tile_ctr, 1u));
+      for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
         const TileRef tr = decode_tile(s, D, t);
         const CUtensorMap* map = tr.is_k ? &a.maps_k[tr.layer] : &a.maps_q[tr.layer];
         const int row0 = tr.idx * 128;
@@ -576,7 +546,6 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
           }
           ++issued;
         }
-        t = next;
       }
       // Every copy still in flight targets this CTA's shared memory: wait for them to land
       // (the latest use of each stage; fp32 v boxes of key stages land on vfull[]).
@@ -596,12 +565,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
       const uint32_t idZ = idesc_f32acc(128, NZ, f16) | (cols ? (1u << 15) : 0u);
       uint32_t consumed = 0, tc = 0, kpar = 0u;
       bool ok = true;
-      for (uint32_t nt = 0; ok; ++nt) {
-        const uint32_t qs = nt % kTileQ;
-        if (!mbar_wait(smem_u32(&tqf[qs]), (nt / kTileQ) & 1u, abort, a.status)) break;
-        const int t = tq[qs];
-        mbar_arrive(smem_u32(&tqe[qs]));
-        if (t >= T) break;
+      for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
         const TileRef tr = decode_tile(s, D, t);
         const uint32_t acc = tc % NA, aph = (tc / NA) & 1u;
         if (!mbar_wait(smem_u32(&acce[acc]), aph ^ 1u, abort, a.status)) break;
@@ -654,13 +618,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     const int gpt = 128 / s.dh;
     const unsigned epoch = FUSED ? __ldcg(a.epoch) : 0u;
     uint32_t tc = 0;
-    for (uint32_t nt = 0;; ++nt) {
-      const uint32_t qs = nt % kTileQ;
-      const bool gotq = mbar_wait(smem_u32(&tqf[qs]), (nt / kTileQ) & 1u, abort, a.status);
-      const int t = gotq ? tq[qs] : T;
-      if (gotq) mbar_arrive(smem_u32(&tqe[qs]));
-      __syncwarp();
-      if (!named_bar_and(4, NE, gotq) || t >= T) break;  // one decision for all epilogue warps
+    for (int t = blockIdx.x; t < T; t += gridDim.x) {
       const TileRef tr = decode_tile(s, D, t);
       const uint32_t acc = tc % NA, aph = (tc / NA) & 1u;
       const bool got = mbar_wait(smem_u32(&accf[acc]), aph, abort, a.status);
@@ -730,13 +688,7 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     const uint32_t ns = static_cast<uint32_t>((s.nkc + BPS - 1) / BPS);  // stages per tile
     uint32_t cnt = 0, kpar = 0u;
     bool ok = true;
-    for (uint32_t nt = 0; ok; ++nt) {
-      const uint32_t qs = nt % kTileQ;
-      const bool gotq = mbar_wait(smem_u32(&tqf[qs]), (nt / kTileQ) & 1u, abort, a.status);
-      const int t = gotq ? tq[qs] : T;
-      if (gotq) mbar_arrive(smem_u32(&tqe[qs]));
-      __syncwarp();
-      if (!named_bar_and(7, NC, gotq) || t >= T) break;  // one decision for both converter warps
+    for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
       const TileRef tr = decode_tile(s, D, t);
       if (!tr.is_k) {  // query tiles: no v operand, only the stage count moves on
         cnt += ns;
@@ -812,15 +764,13 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
   }
   if (FUSED && threadIdx.x == 0) {
     // The last CTA to finish (every CTA gets here, also after giving up on a bounded
-    // wait) clears the per-layer head counts and the tile counter (every CTA's producer
-    // has made its last claim before its CTA got here) and advances the flag epoch for
-    // the next launch; every CTA of this cooperative launch read the epoch at its start, and a
+    // wait) clears the per-layer head counts and advances the flag epoch for the next
+    // launch; every CTA of this cooperative launch read the epoch at its start, and a
     // replayed CUDA graph never takes this launch's flags for its own.
     __threadfence();
     if (atomicAdd(a.done_cnt, 1u) == gridDim.x - 1u) {
       for (int l = 0; l < s.L; ++l) a.layer_cnt[l] = 0u;
       *a.done_cnt = 0u;
-      *a.tile_ctr = 0u;
       const unsigned n = __ldcg(a.epoch) + 1u;
       *a.epoch = n == 0u ? 1u : n;
       __threadfence();

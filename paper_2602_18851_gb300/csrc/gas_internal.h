@@ -119,8 +119,6 @@ struct GramArgs {
   unsigned* layer_cnt;        // [L] finished heads per layer (fused scales), cleared at the end
   unsigned long long* layer_max;  // [L] epoch-tagged maximum sigma bits per layer
   unsigned* done_cnt;         // finished CTAs
-  unsigned* tile_ctr;         // fused variant: tiles handed out past the first wave (dynamic
-                              // schedule); zero at launch, reset by the last CTA
   float* vn2;                 // [L][nq] ||v||^2 summed by the converter warps
   unsigned* vflags;           // [L][tiles_k] v-norm flags (== epoch when vn2 of the tile is ready)
   int iters;
