@@ -267,11 +267,11 @@ def cpu_baseline(wl, iters, budget_s, wq=None, wk=None, v_in=None):
     """The oracle as it stands: the factored form on every host core (the reported value),
     the same form on one core, and the explicit-M form on one head per core."""
     import oracle
-    out = oracle_sample_ms(wl, iters, budget_s, wq=wq, wk=wk, v_in=v_in)
+    nthr = oracle.max_threads()  # read first: a one-thread run changes the pool's default
+    out = oracle_sample_ms(wl, iters, budget_s, wq=wq, wk=wk, v_in=v_in, threads=nthr)
     single = oracle_sample_ms(wl, iters, budget_s / 3, wq=wq, wk=wk, v_in=v_in, threads=1)
-    nthr = oracle.max_threads()
     explicit = oracle_sample_ms(wl, iters, 0.0, wq=wq, wk=wk, v_in=v_in, mode="explicit",
-                                max_heads=min(wl.n_q, nthr))
+                                max_heads=min(wl.n_q, nthr), threads=nthr)
     # heads run in parallel, one per thread: the all-heads estimate divides by the threads
     if min(wl.n_q, nthr) < nthr:
         explicit["value"] *= min(wl.n_q, nthr) / nthr

@@ -90,3 +90,6 @@ def test_cpu_baseline_reports_all_cores_one_core_and_explicit():
     assert c["single_thread"]["cores"] == 1 and c["single_thread"]["value"] > 0
     assert "1 thread" in c["single_thread"]["sample"]
     assert c["explicit"]["value"] > 0 and "explicitly formed" in c["explicit"]["sample"]
+    # the one-thread run leaves the all-core figures alone: the explicit sample uses every core
+    import oracle
+    assert c["explicit"]["cores"] == c["cores"] == oracle.max_threads()
