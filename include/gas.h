@@ -276,8 +276,8 @@ const char *gas_last_launch_name(gas_handle h, int i);
  *   Scratch needed: gas_static_scratch_bytes(layers, d, n_q, d_h), that is, with
  *   nch = ceil(d / 256) and a(x) = x rounded up to a multiple of 256:
  *     2*a(layers*n_q*nch*d_h*4) + 2*a(layers*n_q*nch*4) + 2*a(layers*n_q*d_h*4)
- *     + 3*a(layers*n_q*4) bytes
- *   (17,969,152 bytes for 32 layers, d 4096, 32 heads, d_h 128).  Shapes that need
+ *     + 2*a(layers*n_q*4) bytes
+ *   (17,965,056 bytes for 32 layers, d 4096, 32 heads, d_h 128).  Shapes that need
  *   more than GAS_STATIC_SCRATCH_BYTES are rejected with GAS_ERR_UNSUPPORTED before
  *   any device work.
  *   Errors: as gas_spectral_norms; gas_last_error(NULL) holds the message.
@@ -285,8 +285,8 @@ const char *gas_last_launch_name(gas_handle h, int i);
  * (cudaGetSymbolAddress), so the address stays right after cudaDeviceReset or under
  * another context.  The first call on a device also loads the library's device code:
  * make that first call before any stream capture.  All calls share the array and it
- * keeps the last call's contents; each call clears the part that must start at zero
- * (the reduction counters) on its stream.  Calls whose kernels overlap on the GPU
+ * keeps the last call's contents; every value a call reads from it was written earlier
+ * in the same call, so nothing needs clearing.  Calls whose kernels overlap on the GPU
  * (other streams, other threads) race on the array.
  */
 #define GAS_STATIC_SCRATCH_BYTES (32u * 1024u * 1024u)

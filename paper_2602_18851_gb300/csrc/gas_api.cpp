@@ -44,7 +44,6 @@ struct gas_ctx {
   float* n2r = nullptr;   // [L][nq]
   float* tr = nullptr;    // [L][nq][dh]
   float* s2r = nullptr;   // [L][nq]
-  unsigned* tickets = nullptr;  // [L][nq] last-CTA counters of the streaming passes
   uint16_t* vhl = nullptr;
   float* gq = nullptr;
   float* gk = nullptr;
@@ -252,12 +251,15 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
   a.out2 = h->n2p;
   a.outr = h->zr;
   a.outr2 = h->n2r;
-  a.tickets = h->tickets;
   a.status = h->status;
   a.v_in = v_in;
   a.s_zero = s_out;
   cudaError_t e = launch(h, "stream_pass_k0", st, [&] { return gas::launch_stream_pass(tab, a, st); });
   ++launches;
+  if (e == cudaSuccess) {
+    e = launch(h, "stream_reduce", st, [&] { return gas::launch_stream_reduce(a, st); });
+    ++launches;
+  }
   for (int it = 0; it < iters && e == cudaSuccess; ++it) {
     gas::StreamArgs q{};
     q.s = s;
@@ -269,10 +271,13 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
     q.out2 = h->s2p;
     q.outr = h->tr;
     q.outr2 = h->s2r;
-    q.tickets = h->tickets;
     q.status = h->status;
     e = launch(h, "stream_pass_q", st, [&] { return gas::launch_stream_pass(tab, q, st); });
     ++launches;
+    if (e == cudaSuccess) {
+      e = launch(h, "stream_reduce", st, [&] { return gas::launch_stream_reduce(q, st); });
+      ++launches;
+    }
     if (e != cudaSuccess) break;
     const bool last = (it == iters - 1);
     if (last && v_out == nullptr) break;
@@ -286,12 +291,15 @@ gas_status run_stream(gas_ctx* h, const gas::LayerTable& tab, int iters, const f
     k.out2 = h->n2p;
     k.outr = h->zr;
     k.outr2 = h->n2r;
-    k.tickets = h->tickets;
     k.status = h->status;
     k.v_out = v_out;
     e = launch(h, last ? "stream_pass_kout" : "stream_pass_k", st,
                [&] { return gas::launch_stream_pass(tab, k, st); });
     ++launches;
+    if (e == cudaSuccess) {
+      e = launch(h, "stream_reduce", st, [&] { return gas::launch_stream_reduce(k, st); });
+      ++launches;
+    }
   }
   if (e == cudaSuccess) {
     gas::FinalizeArgs f{};
@@ -577,7 +585,6 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   const size_t o_n2r = take(L * NQ * 4);
   const size_t o_tr = take(L * NQ * DH * 4);
   const size_t o_s2r = take(L * NQ * 4);
-  const size_t o_tickets = take(L * NQ * sizeof(unsigned));
   const size_t o_vhl = take(L * s.tiles_k * static_cast<size_t>(s.nz) * d * 2);
   const size_t o_gq = take(L * s.tiles_q * 16384ull * 4);
   const size_t o_gk = take(L * s.tiles_k * 16384ull * 4);
@@ -615,7 +622,6 @@ gas_status gas_create(int layers, int d, int n_q, int n_kv, int d_h, gas_handle*
   h->n2r = reinterpret_cast<float*>(b + o_n2r);
   h->tr = reinterpret_cast<float*>(b + o_tr);
   h->s2r = reinterpret_cast<float*>(b + o_s2r);
-  h->tickets = reinterpret_cast<unsigned*>(b + o_tickets);
   h->vhl = reinterpret_cast<uint16_t*>(b + o_vhl);
   h->gq = reinterpret_cast<float*>(b + o_gq);
   h->gk = reinterpret_cast<float*>(b + o_gk);

@@ -52,9 +52,9 @@ __host__ __device__ inline long long weight_row_offset(int r, int dh, long long 
 // ---- streaming matvec-chain passes (Algorithm 2 applied literally) ---------------
 // One pass streams one weight matrix X (a head's A_h or a group's B_g, d_h x d) in
 // column chunks.  For every vector that uses X it forms p = X^T x over the chunk
-// (and ||p||^2), then either q = X p (partial over the chunk) or writes p out.  The
-// last chunk CTA of every matrix sums the chunk partials (in chunk order) into one
-// d_h-vector and one squared norm per head, which the next pass reads.
+// (and ||p||^2), then either q = X p (partial over the chunk) or writes p out.  A short
+// reduction kernel then sums the chunk partials (in chunk order) into one d_h-vector and
+// one squared norm per head, which the next pass reads.
 enum StreamMode : int {
   kPassQ = 0,      // X = A_h, x = z / ||v'|| (K results); out: t = A_h u', ||u'||^2
   kPassK = 1,      // X = B_g, x = t / ||u'|| = y (Q results, G heads); out: z = B_g v', ||v'||^2
@@ -72,7 +72,6 @@ struct StreamArgs {
   float* out2;        // [L][nq][nch]     ||p||^2 partials            (all modes)
   float* outr;        // [L][nq][dh]      q summed over the chunks    (modes Q, K, K0)
   float* outr2;       // [L][nq]          ||p||^2 summed over the chunks (all modes)
-  unsigned* tickets;  // [L][nq] chunk counters of the last-CTA reduction; zero between passes
   const float* v_in;  // [L][nq][d]                                   (mode K0)
   float* v_out;       // [L][nq][d]                                   (mode KOut)
   float* s_zero;      // mode K0: per-layer scale slots zeroed for the fused epilogue
@@ -189,6 +188,7 @@ inline cudaError_t set_smem_per_device(const void* kernel, int bytes, unsigned l
 
 // Launchers (return cudaGetLastError() of the launch).
 cudaError_t launch_stream_pass(const LayerTable& tab, const StreamArgs& a, cudaStream_t st);
+cudaError_t launch_stream_reduce(const StreamArgs& a, cudaStream_t st);  // chunk sums of a pass
 cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st);
 cudaError_t launch_scales(const ScalesArgs& a, cudaStream_t st);
 cudaError_t launch_prep_v(const PrepArgs& a, cudaStream_t st);

@@ -36,9 +36,8 @@ size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 cudaError_t static_scratch_ptr(void** out) { return cudaGetSymbolAddress(out, g_static_scratch); }
 
 // Bytes of scratch one call needs (0 for sizes that are not positive).
-// Layout: z and t partials [L][n_q][nch][d_h], their squared-norm partials [L][n_q][nch],
-// the chunk sums of both ([L][n_q][d_h] and [L][n_q]) and the passes' ticket counters
-// [L][n_q], each region 256-byte aligned.
+// Layout: z and t partials [L][n_q][nch][d_h], their squared-norm partials [L][n_q][nch]
+// and the chunk sums of both ([L][n_q][d_h] and [L][n_q]), each region 256-byte aligned.
 struct StaticLayout {
   size_t vec, nrm, rvec, rnrm, total;
 };
@@ -50,7 +49,7 @@ StaticLayout static_layout(int layers, int d, int n_q, int d_h) {
   o.nrm = static_cast<size_t>(layers) * n_q * nch * sizeof(float);
   o.rvec = static_cast<size_t>(layers) * n_q * d_h * sizeof(float);
   o.rnrm = static_cast<size_t>(layers) * n_q * sizeof(float);
-  o.total = 2 * align256(o.vec) + 2 * align256(o.nrm) + 2 * align256(o.rvec) + 3 * align256(o.rnrm);
+  o.total = 2 * align256(o.vec) + 2 * align256(o.nrm) + 2 * align256(o.rvec) + 2 * align256(o.rnrm);
   return o;
 }
 
@@ -116,19 +115,10 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
   float* tr = reinterpret_cast<float*>(r + gas::align256(rvec));
   float* n2r = reinterpret_cast<float*>(r + 2 * gas::align256(rvec));
   float* s2r = reinterpret_cast<float*>(r + 2 * gas::align256(rvec) + gas::align256(rnrm));
-  unsigned* tickets = reinterpret_cast<unsigned*>(r + 2 * gas::align256(rvec) + 2 * gas::align256(rnrm));
-  // Every scratch element a pass reads was written earlier in the same call (each pass
-  // covers all heads, chunks and rows), except the ticket counters of the last-CTA
-  // reductions: those must start at zero.  Where they sit depends on the shape, so an
-  // earlier call with another shape may have left partial sums there; they are cleared
-  // on the stream at the start of every call (every pass leaves them at zero again).
+  // Every scratch value a pass reads was written earlier in the same call (each pass and
+  // its chunk reduction cover all heads, chunks and rows), so nothing carries over from
+  // an earlier call and nothing has to be cleared.
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  e = cudaMemsetAsync(tickets, 0, gas::align256(rnrm), st);
-  if (e != cudaSuccess) {
-    snprintf(buf, sizeof(buf), "gas_spectral_norms_static: clearing the ticket counters failed: %s",
-             cudaGetErrorString(e));
-    return static_fail(GAS_ERR_CUDA, buf);
-  }
 
   gas::LayerTable tab;
   std::memset(&tab, 0, sizeof(tab));
@@ -143,9 +133,9 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
   a.out2 = n2p;
   a.outr = zr;
   a.outr2 = n2r;
-  a.tickets = tickets;
   a.v_in = v_in;
   e = gas::launch_stream_pass(tab, a, st);
+  if (e == cudaSuccess) e = gas::launch_stream_reduce(a, st);
   for (int it = 0; it < iters && e == cudaSuccess; ++it) {
     gas::StreamArgs q{};
     q.s = s;
@@ -157,8 +147,8 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
     q.out2 = s2p;
     q.outr = tr;
     q.outr2 = s2r;
-    q.tickets = tickets;
     e = gas::launch_stream_pass(tab, q, st);
+    if (e == cudaSuccess) e = gas::launch_stream_reduce(q, st);
     const bool last = (it == iters - 1);
     if (e != cudaSuccess || (last && v_out == nullptr)) break;
     gas::StreamArgs k{};
@@ -171,9 +161,9 @@ extern "C" gas_status gas_spectral_norms_static(int layers, int d, int n_q, int 
     k.out2 = n2p;
     k.outr = zr;
     k.outr2 = n2r;
-    k.tickets = tickets;
     k.v_out = v_out;
     e = gas::launch_stream_pass(tab, k, st);
+    if (e == cudaSuccess) e = gas::launch_stream_reduce(k, st);
   }
   if (e == cudaSuccess) {
     gas::FinalizeArgs f{};

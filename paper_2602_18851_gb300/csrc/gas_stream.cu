@@ -10,10 +10,9 @@
 // Each CTA streams one d_h x 256 weight tile (bf16, binary16 or fp32; any d_h in
 // {64, 80, 96, 128, 256}) with 16-byte loads, issued before anything else, and stages
 // its input vectors (one, or the G of a key group) in shared memory while they land.
-// Its results over its columns go to a small fp32 workspace indexed by chunk; the last
-// CTA of each matrix to finish (a ticket counter) sums them in chunk order into one
-// d_h-vector and one squared norm per head.  No float atomics: results are
-// deterministic.
+// Its results over its columns go to a small fp32 workspace indexed by chunk; a second,
+// short kernel sums them in chunk order into one d_h-vector and one squared norm per
+// head.  No float atomics: results are deterministic.
 
 #include "gas_device.cuh"
 
@@ -59,7 +58,6 @@ __global__ void __launch_bounds__(32 * stream_warps(DH), (WT == kWF32 || DH > 12
   __shared__ __align__(16) float xs[kStreamVB][DH];
   __shared__ __align__(16) float red[NW][kStreamChunk];
   __shared__ __align__(16) float ps[kStreamChunk];
-  __shared__ unsigned is_last;
 
   const int nvec = (MODE == kPassQ) ? 1 : s.G;
   const size_t h0 = static_cast<size_t>(l) * s.nq + ((MODE == kPassQ) ? m : m * s.G);  // head of vector 0
@@ -149,42 +147,39 @@ __global__ void __launch_bounds__(32 * stream_warps(DH), (WT == kWF32 || DH > 12
     }
   }
   if (MODE == kPassK0 && a.s_zero != nullptr && chunk == 0 && m == 0 && tid == 0) a.s_zero[l] = 0.0f;
+}
 
-  // The last chunk CTA of this matrix sums every vector's chunk partials, in chunk order.
-  __threadfence();
-  __syncthreads();
-  unsigned* ticket = a.tickets + static_cast<size_t>(l) * gridDim.y + m;
-  if (tid == 0) is_last = (atomicAdd(ticket, 1u) + 1u == gridDim.x) ? 1u : 0u;
-  __syncthreads();
-  if (!is_last) return;
-  __threadfence();
+// Sums of the chunk partials of a pass, in chunk order: outr[h] = sum_c out[h][c] (modes Q,
+// K, K0) and outr2[h] = sum_c out2[h][c] (all modes), one thread per output value.  A
+// separate launch: the pass's CTAs write their partials and exit without a fence or a
+// ticket, so none of them waits for its stores to be acknowledged.
+template <int DH>
+__global__ void __launch_bounds__(256) stream_reduce_kernel(const __grid_constant__ StreamArgs a) {
+  const Shape& s = a.s;
+  const size_t heads = static_cast<size_t>(s.L) * s.nq;
   const int nch = s.nch;
-  if (MODE != kPassKOut) {
-    for (int i = tid; i < nvec * DH; i += NT) {
-      const int jj = i / DH, r = i - jj * DH;
-      const size_t hidx = h0 + jj;
-      const float* src = a.out + hidx * nch * DH + r;
-      float acc[8];
+  const size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (a.mode != kPassKOut && i < heads * DH) {
+    const size_t hidx = i / DH, r = i - hidx * DH;
+    const float* src = a.out + hidx * nch * DH + r;
+    float acc[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
-      for (int c0 = 0; c0 < nch; c0 += 8) {  // eight loads in flight per step
-        float t[8];
+    for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
+    for (int c0 = 0; c0 < nch; c0 += 8) {  // eight loads in flight per step
+      float t[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) t[e] = c0 + e < nch ? __ldcg(src + static_cast<size_t>(c0 + e) * DH) : 0.0f;
+      for (int e = 0; e < 8; ++e) t[e] = c0 + e < nch ? __ldcg(src + static_cast<size_t>(c0 + e) * DH) : 0.0f;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[e] += t[e];
-      }
-      a.outr[hidx * DH + r] = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+      for (int e = 0; e < 8; ++e) acc[e] += t[e];
     }
+    a.outr[i] = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
   }
-  for (int jj = warp; jj < nvec; jj += NW) {
-    const size_t hidx = h0 + jj;
+  if (i < heads) {
+    const float* src = a.out2 + i * nch;
     float v = 0.0f;
-    for (int c = lane; c < nch; c += 32) v += __ldcg(a.out2 + hidx * nch + c);
-    v = warp_sum(v);
-    if (lane == 0) a.outr2[hidx] = v;
+    for (int c = 0; c < nch; ++c) v += __ldcg(src + c);
+    a.outr2[i] = v;
   }
-  if (tid == 0) *ticket = 0u;
 }
 
 // sigma = ||u'|| of the last Q pass; v_out = v' / ||v'|| of the last K pass; fused
@@ -256,6 +251,21 @@ cudaError_t launch_stream_pass(const LayerTable& tab, const StreamArgs& a, cudaS
     case 256: return launch_stream_dh<256>(tab, a, st);
     default: return cudaErrorInvalidValue;
   }
+}
+
+cudaError_t launch_stream_reduce(const StreamArgs& a, cudaStream_t st) {
+  const int dh = a.s.dh;
+  const size_t outs = static_cast<size_t>(a.s.L) * a.s.nq * (a.mode == kPassKOut ? 1 : dh);
+  const unsigned grid = static_cast<unsigned>((outs + 255) / 256);
+  switch (dh) {
+    case 64: stream_reduce_kernel<64><<<grid, 256, 0, st>>>(a); break;
+    case 80: stream_reduce_kernel<80><<<grid, 256, 0, st>>>(a); break;
+    case 96: stream_reduce_kernel<96><<<grid, 256, 0, st>>>(a); break;
+    case 128: stream_reduce_kernel<128><<<grid, 256, 0, st>>>(a); break;
+    case 256: stream_reduce_kernel<256><<<grid, 256, 0, st>>>(a); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st) {
