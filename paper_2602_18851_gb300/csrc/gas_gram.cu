@@ -502,6 +502,11 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
     // ---------------- TMA producer ----------------
     if (lane == 0) {
       const uint64_t pol = l2_policy_evict_first();
+      // The key tiles of the last layers stay in L2 (evict_last) for the write-back, which
+      // walks the layers from the last one down: about 48 MB of them.
+      const uint64_t pol_k = l2_policy_evict_last();
+      const long long kbytes = static_cast<long long>(s.tiles_k) * 128 * s.d * 2;
+      const int keep0 = s.L - static_cast<int>(max(1LL, (48LL << 20) / kbytes));
       uint32_t issued = 0, kpar = 0u, kmask = 0u;  // kmask bit st: the latest use of st was a key stage
       bool ok = true;
       for (int t = blockIdx.x; t < T && ok; t += gridDim.x) {
@@ -530,7 +535,8 @@ __global__ void __launch_bounds__(GramWarps<FUSED>::kThreads, 1) gram_kernel(con
               tma_load_2d(bx, map, fb, row0, (kc + b) * 64, pol);
               tma_load_2d(bx + kTileBytes / 2, map, fb, row0 + 64, (kc + b) * 64, pol);
             } else {
-              tma_load_3d(bx, map, fb, (kc + b) * 64, 0, row0 / DH, pol);  // 128/d_h heads of d_h rows
+              tma_load_3d(bx, map, fb, (kc + b) * 64, 0, row0 / DH,  // 128/d_h heads of d_h rows
+                          tr.is_k && tr.layer >= keep0 ? pol_k : pol);
             }
             if (tr.is_k) {
               if (FUSED)  // fp32 rows of the tile's heads: layer * nq + first head of the tile

@@ -44,11 +44,14 @@ struct WbItem {
   int layer, tile, c0, nchunks;
 };
 
+// Items walk the layers from the last one down: the Gram launch read the key tiles of
+// its last layers most recently (and keeps them in L2), so the first items hit L2.
 __device__ __forceinline__ WbItem decode_item(const Shape& s, int t) {
   const int ncb = (s.d + kWbCols - 1) / kWbCols;
   WbItem w;
-  w.layer = t / (s.tiles_k * ncb);
-  const int rem = t - w.layer * s.tiles_k * ncb;
+  const int lr = t / (s.tiles_k * ncb);
+  w.layer = s.L - 1 - lr;
+  const int rem = t - lr * s.tiles_k * ncb;
   w.tile = rem / ncb;
   w.c0 = (rem - w.tile * ncb) * kWbCols;
   const int ncols = min(kWbCols, s.d - w.c0);
