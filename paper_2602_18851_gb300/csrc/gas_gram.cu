@@ -19,7 +19,11 @@
 //                   which also sum ||v||^2 per head; its epilogue runs the k iterations
 //   iterate_kernel  (unfused) k iterations per head in R^{d_h} from G_Q, G_K, z0; sigma,
 //                   y/||v'||, fused per-layer scale (Eq. 15)
-// The write-back v_out = B^T y / ||v'|| is its own tensor-core kernel (gas_writeback.cu).
+// The write-back v_out = B^T y / ||v'|| is its own tensor-core kernel (gas_writeback.cu),
+// launched as a programmatic dependent of this one: every CTA here signals it once its
+// prologue is done, so the write-back's CTAs can set up and prefetch W^K on the SMs this
+// launch leaves.  The key tiles of the last layers are read with an L2 evict-last policy,
+// because the write-back starts with those layers.
 
 #include "gas_device.cuh"
 
