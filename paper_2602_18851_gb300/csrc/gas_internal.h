@@ -76,6 +76,7 @@ struct StreamArgs {
   float* v_out;       // [L][nq][d]                                   (mode KOut)
   float* s_zero;      // mode K0: per-layer scale slots zeroed for the fused epilogue
   unsigned* status;   // device status word (may be null)
+  long long pf_dist;  // streaming pass: CTAs ahead whose tile is prefetched into L2 (0: none)
 };
 
 struct FinalizeArgs {

@@ -12,7 +12,8 @@
 // its input vectors (one, or the G of a key group) in shared memory while they land.
 // Its results over its columns go to a small fp32 workspace indexed by chunk; a second,
 // short kernel sums them in chunk order into one d_h-vector and one squared norm per
-// head.  No float atomics: results are deterministic.
+// head.  No float atomics: results are deterministic.  In a Q pass every CTA also
+// prefetches into L2 the tile of the CTA one wave after it, which then loads from L2.
 
 #include "gas_device.cuh"
 
@@ -53,6 +54,29 @@ __global__ void __launch_bounds__(32 * stream_warps(DH), (WT == kWF32 || DH > 12
   for (int rr = 0; rr < R; ++rr) {
     const int row = warp + NW * rr;
     w[rr] = (rr < RV && colok) ? load_w8<WT>(X, x0 + static_cast<long long>(row) * ld + col) : zero_w8<WT>();
+  }
+  // Bring into L2 the tile of the CTA a.pf_dist positions later in launch order (about one
+  // wave ahead): when that CTA runs, its loads hit L2, so a CTA spends less of its life
+  // waiting and more of the SM's time has weights in flight.
+  if (a.pf_dist > 0) {
+    const long long lin = blockIdx.x + static_cast<long long>(gridDim.x) * (blockIdx.y + static_cast<long long>(gridDim.y) * blockIdx.z);
+    const long long fut = lin + a.pf_dist;
+    const long long total = static_cast<long long>(gridDim.x) * gridDim.y * gridDim.z;
+    if (fut < total) {
+      const int fc = static_cast<int>(fut % gridDim.x);
+      const long long fr = fut / gridDim.x;
+      const int fm = static_cast<int>(fr % gridDim.y), fl = static_cast<int>(fr / gridDim.y);
+      const int fcol = fc * kStreamChunk + lane * 8;
+      if (fcol < s.d) {
+        const char* FX = reinterpret_cast<const char*>((MODE == kPassQ) ? tab.q[fl] : tab.k[fl]);
+        const long long fx0 = static_cast<long long>(fm) * hstride;
+#pragma unroll
+        for (int rr = 0; rr < RV; ++rr) {
+          const long long e = fx0 + static_cast<long long>(warp + NW * rr) * ld + fcol;
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(FX + e * (WT == kWF32 ? 4 : 2)));
+        }
+      }
+    }
   }
 
   __shared__ __align__(16) float xs[kStreamVB][DH];
@@ -217,8 +241,24 @@ __global__ void __launch_bounds__(32) scales_kernel(const __grid_constant__ Scal
   if (threadIdx.x == 0) a.s[l] = a.scale_c * m;
 }
 
+// Streaming multiprocessors of the current device (looked up once per device).
+int current_sm_count() {
+  static int counts[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
+  if (dev < 64 && __atomic_load_n(&counts[dev], __ATOMIC_RELAXED) > 0) return __atomic_load_n(&counts[dev], __ATOMIC_RELAXED);
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  if (dev < 64) __atomic_store_n(&counts[dev], n, __ATOMIC_RELAXED);
+  return n;
+}
+
 template <int DH, int WT>
-cudaError_t launch_stream_dt(const LayerTable& tab, const StreamArgs& a, cudaStream_t st) {
+cudaError_t launch_stream_dt(const LayerTable& tab, const StreamArgs& a_in, cudaStream_t st) {
+  // Q passes (one vector per tile, bound by the weight stream) prefetch the tile of the CTA
+  // one wave later into L2; key passes (G vectors per tile, bound by the SM) do not.
+  StreamArgs a = a_in;
+  a.pf_dist = a.mode == kPassQ ? static_cast<long long>(current_sm_count()) * ((WT == kWF32 || DH > 128) ? 1 : 2) : 0;
   const dim3 block(32 * stream_warps(DH));
   const dim3 grid(a.s.nch, a.mode == kPassQ ? a.s.nq : a.s.nkv, a.s.L);
   switch (a.mode) {
